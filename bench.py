@@ -1,0 +1,408 @@
+#!/usr/bin/env python
+"""Throughput of the energy-guided cached DiT step on GB300.
+
+One step = one pass of the whole hot path over one batch of synthetic input:
+audio segment energy, then per layer the energy-guided selection (drift score
++ top-K) and the block on the selected latents (gather, self-attention with
+K/V over all latents, cross-attention to the audio tokens, FFN, int8 cache
+write, merge).  Default workload: one Wan2.2-S2V-shaped block, 21x30x52 =
+32760 latent tokens, D 5120, 40 heads x 128, FFN 13824, 672 audio tokens,
+refresh ratio 1/5 (6552 active tokens), synthetic speech-like audio,
+random-init weights.
+
+Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle on
+the host cores instead (a bounded sample of the same step, extrapolated).
+Multi-GPU: independent replicas (the step does not shard; no collective on
+the data path); value = tokens of all ranks / max rank time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "cached DiT step latent tokens/s"
+UNIT = "tokens/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="wan_block_32760")
+    ap.add_argument("--ratio", default=None, help="num/den refresh ratio override")
+    ap.add_argument("--profile", default="audio", help="audio profile")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples during the timed region."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index, self.lines, self.proc = index, [], None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            threading.Thread(target=self._read, daemon=True).start()
+        except (OSError, ValueError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, mx, reasons = [], None, set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            p = [x.strip() for x in ln.split(",")]
+            if len(p) < 8:
+                continue
+            try:
+                sm.append(float(p[0]))
+                mx = float(p[1])
+            except ValueError:
+                continue
+            for nm, v in zip(names, p[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+def algorithmic_work(name, m, n, k, K, xbytes=2):
+    """(flops, bytes) one launch must do, from its recorded shape."""
+    if name == "gemm_tcgen05":
+        return 2.0 * m * n * k, None
+    if name == "attention":
+        return 4.0 * m * n * k, None
+    if name == "drift_score":
+        return None, m * n * (xbytes + 1) + 8.0 * m
+    if name == "dequant_merge":
+        NT, D = m, n
+        return None, (NT - K) * (D + 4) + K * 2 * D + NT * 2 * D + 4 * NT
+    if name == "quant_scatter":
+        return None, m * n * 3 + 8.0 * m
+    if name == "layernorm_gather":
+        return None, m * n * 4
+    return None, None
+
+
+def roofline(records, K, peaks):
+    agg = {}
+    for name, m, n, k, ms in records:
+        a = agg.setdefault((name, m, n, k), [0, 0.0])
+        a[0] += 1
+        a[1] += ms
+    by_kernel = {}
+    for (name, m, n, k), (cnt, ms) in agg.items():
+        b = by_kernel.setdefault(name, [0, 0.0])
+        b[0] += cnt
+        b[1] += ms
+    total = sum(v[1] for v in by_kernel.values())
+    dom = max(by_kernel, key=lambda x: by_kernel[x][1])
+    # the dominant kernel's largest launch shape (most time)
+    shapes = [(ms / cnt, cnt, key) for key, (cnt, ms) in agg.items() if key[0] == dom]
+    shape = max(shapes, key=lambda s: s[0] * s[1])
+    avg_ms, cnt, (name, m, n, k) = shape
+    flops, byts = algorithmic_work(name, m, n, k, K)
+    if flops is not None:
+        achieved = flops / (avg_ms * 1e-3) / 1e12
+        peak = peaks["bf16_tflops_sustained"]
+        out = {"bound": "tensor", "kernel": name, "shape": [m, n, k], "achieved": round(achieved, 2),
+               "peak": peak, "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
+               "traffic": None, "algorithmic_flops": flops, "launch_ms": round(avg_ms, 4),
+               "peak_source": "measured bf16_tflops_sustained"}
+    else:
+        achieved = byts / (avg_ms * 1e-3) / 1e9
+        peak = peaks["hbm_gbs"]
+        out = {"bound": "hbm", "kernel": name, "shape": [m, n, k], "achieved": round(achieved, 1),
+               "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": None,
+               "algorithmic_bytes": byts, "launch_ms": round(avg_ms, 4),
+               "peak_source": "measured hbm_gbs"}
+    table = {}
+    for (nm, m, n, k), (c, ms) in sorted(agg.items(), key=lambda kv: -kv[1][1]):
+        f, b = algorithmic_work(nm, m, n, k, K)
+        row = {"launches": c, "ms_per_launch": round(ms / c, 4), "share": round(ms / total, 4)}
+        if f is not None:
+            row["tflops"] = round(f / (ms / c * 1e-3) / 1e12, 1)
+        if b is not None:
+            row["gbs"] = round(b / (ms / c * 1e-3) / 1e9, 1)
+        table[f"{nm}[{m}x{n}x{k}]"] = row
+    return out, table
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d["bf16_tflops_sustained"], "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
+
+
+# ---------------------------------------------------------------------------
+def oracle_sample(w, audio, W, cond, x1, q, s, rnum, rden, budget_s=25.0):
+    """Time the CPU oracle on a bounded sample of one cached step and extrapolate.
+
+    Measured in full: audio energy, drift + top-K over all tokens, the merge
+    (reconstruction of the inactive rows) and the int8 write of the active rows.
+    Sampled: K/V projection of `s_kv` rows (scaled by NT / s_kv) and the
+    active-row block (Q', attention over all NT keys, cross-attention, FFN) of
+    `s_a` rows (scaled by K / s_a)."""
+    import numpy as np
+    import oracle
+    t = {}
+    t0 = time.perf_counter()
+    _, e = oracle.energy.audio_energy(audio, w.T)
+    t["energy"] = time.perf_counter() - t0
+    e32 = e.astype(np.float32)
+    t0 = time.perf_counter()
+    idx, _ = oracle.select.select(x1, q, s, e32, w.T, w.N, rnum, rden)
+    t["select"] = time.perf_counter() - t0
+    K = len(idx)
+    s_kv = min(w.NT, 1024)
+    t0 = time.perf_counter()
+    oracle.block.self_kv(x1[:s_kv], W)
+    t["kv_sample"] = time.perf_counter() - t0
+    Kc, Vc = oracle.block.cross_kv(cond, W)
+    kv_stand_in = x1.astype(np.float64)      # any [NT, D] array: only the timing is used
+    s_a = min(K, 32)
+    t0 = time.perf_counter()
+    oracle.block.active_rows(x1, idx[:s_a], W, w.H, kv_stand_in, kv_stand_in, Kc, Vc)
+    t["active_sample"] = time.perf_counter() - t0
+    inactive = np.setdiff1d(np.arange(w.NT), idx)
+    t0 = time.perf_counter()
+    oracle.cache.dequantize_rows(q[inactive], s[inactive])
+    qq, ss = q.copy(), s.copy()
+    oracle.cache.quant_scatter(x1[idx], idx, qq, ss)
+    t["merge_quant"] = time.perf_counter() - t0
+    per_layer = (t["select"] + t["kv_sample"] * w.NT / s_kv + t["active_sample"] * K / s_a
+                 + t["merge_quant"])
+    step_s = t["energy"] + w.layers * per_layer
+    sample = (f"oracle on one {w.name} cached step: energy, drift+top-K over all {w.NT} tokens, "
+              f"merge and int8 write in full; K/V projection timed on {s_kv} of {w.NT} rows and "
+              f"the active-row block on {s_a} of {K} rows, each scaled to the full count; "
+              f"one layer timed, times {w.layers} layers; {sum(t.values()):.1f} s of CPU time")
+    return step_s, sample, t
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+# ---------------------------------------------------------------------------
+def build_inputs(w, profile):
+    import numpy as np
+    from synth import generate as G
+    audio = G.audio(w, profile)
+    W = G.block_weights(w, 0)
+    cond = G.cond_tokens(w, audio)
+    x0 = G.latents(w)
+    xs = [G.step_input(w, x0, t) for t in (1, 2)]
+    return audio, W, cond, x0, xs
+
+
+def run_reference(args, w, rnum, rden, rank):
+    if rank != 0:
+        return
+    import numpy as np
+    import oracle
+    audio, W, cond, x0, xs = build_inputs(w, args.profile)
+    q, s, _ = oracle.cache.quantize_rows(x0)
+    times = []
+    for i in range(args.warmup + args.steps):
+        step_s, sample, _ = oracle_sample(w, audio, W, cond, xs[i % 2], q, s, rnum, rden)
+        if i >= args.warmup:
+            times.append(step_s)
+    ms = 1e3 * statistics.mean(times)
+    val = w.NT / (ms * 1e-3)
+    line = {"impl": "reference", "metric": METRIC, "value": round(val, 2), "unit": UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(ms, 2), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "tokens": w.NT, "D": w.D, "heads": f"{w.H}x{w.d}",
+                       "ffn": w.F, "audio_tokens": w.Lc, "ratio": f"{rnum}/{rden}",
+                       "layers": w.layers},
+            "cpu_baseline": {"value": round(val, 2), "unit": UNIT, "cores": cpu_cores(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(val, 2), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    from synth import ALL
+    w = ALL[args.workload]
+    rnum, rden = (w.ratio_num, w.ratio_den)
+    if args.ratio:
+        rnum, rden = (int(v) for v in args.ratio.split("/"))
+    args.profile = "speech" if args.profile == "audio" else args.profile
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, w, rnum, rden, rank)
+        return
+
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+    from paper_2608_02474_gb300 import echocache as ec
+    from paper_2608_02474_gb300.pipeline import CachedStack
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    audio, W, cond, x0, xs = build_inputs(w, args.profile)
+    blocks = [ec.DeviceBlock.from_host(W, cond, device=dev) for _ in range(w.layers)]
+    stack = CachedStack(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc, blocks, device=dev)
+    audio_d = torch.from_numpy(audio).to(dev)
+    x0_d = torch.from_numpy(x0).to(dev, torch.bfloat16)
+    xs_d = [torch.from_numpy(x).to(dev, torch.bfloat16) for x in xs]
+    stack.set_audio(audio_d)
+    stack.step(x0_d, 1, 1, full=True)          # fills every layer's cache (untimed setup)
+    K = w.K if (rnum, rden) == (w.ratio_num, w.ratio_den) else (rnum * w.NT + rden - 1) // rden
+
+    def one_step(x):
+        stack.set_audio(audio_d)
+        return stack.step(x, rnum, rden)
+
+    for i in range(args.warmup):
+        one_step(xs_d[i % 2])
+    torch.cuda.synchronize()
+    assert ec.echo_get_device_error() == 0
+
+    # ---- device-timed region: inputs resident in HBM ----
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    stream = torch.cuda.current_stream()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize()
+    l0 = ec.echo_launch_count()
+    ev0.record(stream)
+    for i in range(args.steps):
+        one_step(xs_d[i % 2])
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    launches = ec.echo_launch_count() - l0
+    clk = clocks.stop()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    assert ec.echo_get_device_error() == 0
+    value = world * w.NT / (ms * 1e-3)
+
+    # ---- per-kernel times: the same steps again with every launch bracketed by events ----
+    ec.echo_profile_enable(True)
+    for i in range(args.steps):
+        one_step(xs_d[i % 2])
+    torch.cuda.synchronize()
+    ec.echo_profile_enable(False)
+    records = ec.echo_profile_read()
+    peaks = load_peaks()
+    roof, table = roofline(records, K, peaks)
+
+    # ---- end to end through the public API with host buffers ----
+    e2e = None
+    if not args.no_e2e:
+        xh = [torch.from_numpy(x).to(torch.bfloat16).pin_memory() for x in xs]
+        yh = torch.empty(w.NT, w.D, dtype=torch.bfloat16).pin_memory()
+        xd = torch.empty(w.NT, w.D, dtype=torch.bfloat16, device=dev)
+        for i in range(2):
+            xd.copy_(xh[i % 2], non_blocking=True)
+            yh.copy_(one_step(xd), non_blocking=True)
+        torch.cuda.synchronize()
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(args.steps):
+            xd.copy_(xh[i % 2], non_blocking=True)
+            yh.copy_(one_step(xd), non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        ems = e0.elapsed_time(e1) / args.steps
+        if world > 1:
+            t = torch.tensor([ems], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ems = float(t.item())
+        e2e = {"value": round(world * w.NT / (ems * 1e-3), 2), "unit": UNIT,
+               "h2d_bytes_per_step": xh[0].numel() * 2, "d2h_bytes_per_step": yh.numel() * 2,
+               "ms_per_step": round(ems, 3)}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        q, s, _ = oracle.cache.quantize_rows(x0)
+        step_s, sample, _ = oracle_sample(w, audio, W, cond, xs[0], q, s, rnum, rden)
+        cpu = {"value": round(w.NT / step_s, 2), "unit": UNIT, "cores": cpu_cores(),
+               "kind": "oracle", "sample": sample, "ms_per_step": round(step_s * 1e3, 1)}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "bf16", "data": "synthetic",
+                "config": {"workload": w.name, "tokens": w.NT, "active_tokens": K,
+                           "ratio": f"{rnum}/{rden}", "D": w.D, "heads": f"{w.H}x{w.d}",
+                           "ffn": w.F, "audio_tokens": w.Lc, "layers": w.layers,
+                           "audio": args.profile, "parallelism": f"replicas{world}",
+                           "l2": "inputs larger than L2 (x 335 MB, weights 702 MB per block)"},
+                "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+                "gpu_launches": launches, "kernels": table}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,276 @@
+/*
+ * echocache.h - C ABI of the energy-guided cached DiT step (EchoCache,
+ * arXiv 2608.02474), GB300 (sm_103a) build.
+ *
+ * One cached step of one DiT layer, in the paper's order:
+ *   echo_audio_energy  - audio -> per-segment time-frequency energy
+ *                        (Sec. 3.3 "Cross-modal Saliency Anchors")
+ *   echo_select        - per-token drift (Eq. 1, per token) weighted by segment
+ *                        energy, top-K -> ascending active index list
+ *                        (Sec. 3.3, budget k_t = ceil(N r_t) read globally)
+ *   echo_block_step    - the block on the active latents: Q' on active, K/V on
+ *                        all latents, cross-attention, FFN on active, merge with
+ *                        the cache, write the active rows back to the cache
+ *                        (Sec. 3.3 "Fine-grained latent-level caching",
+ *                        Sec. 3.4 for the int8 cache)
+ *   echo_cache_quant / echo_cache_dequant - the int8 per-token cache (Sec. 3.4)
+ *
+ * Conventions (every entry point):
+ *   - All tensor pointers are DEVICE pointers unless stated; all tensors are
+ *     row-major and contiguous, batch 1.  bf16 is IEEE bfloat16 (2 bytes).
+ *   - The caller allocates and owns every buffer, workspace and the stream.
+ *     The library never allocates device memory and never synchronises the
+ *     host, except echo_get_device_error.
+ *   - Work is enqueued on `stream` (NULL = legacy default stream) and is
+ *     stream-ordered; buffers must stay valid until the stream has run it.
+ *   - Arguments are checked before anything is enqueued: a bad argument
+ *     returns an error and enqueues nothing.  Device pointers must be 16-byte
+ *     aligned.  A launch failure returns ECHO_ERR_CUDA.
+ *   - Data-dependent errors (a non-finite amax or score, a bounded device wait
+ *     that gave up) set a device-side flag; echo_get_device_error reports and
+ *     clears it.  No kernel traps.
+ *   - Thread safety: calls may come from several host threads; calls on one
+ *     stream run in order.
+ */
+#ifndef ECHOCACHE_H
+#define ECHOCACHE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same object as cudaStream_t. */
+typedef struct CUstream_st *echo_stream_t;
+
+typedef enum {
+    ECHO_OK = 0,
+    ECHO_ERR_INVALID_ARG = 1,  /* null pointer, misaligned pointer, bad enum */
+    ECHO_ERR_SHAPE = 2,        /* unsupported or inconsistent sizes */
+    ECHO_ERR_WORKSPACE = 3,    /* workspace smaller than the size query */
+    ECHO_ERR_CUDA = 4,         /* a CUDA call or launch failed */
+    ECHO_ERR_NONFINITE = 5,    /* device flag: NaN/Inf met in a score or amax */
+    ECHO_ERR_TIMEOUT = 6,      /* device flag: a bounded device wait gave up */
+    ECHO_ERR_UNSUPPORTED = 7   /* no sm_103a device */
+} echo_status;
+
+typedef enum { ECHO_BF16 = 0, ECHO_F32 = 1 } echo_dtype;
+
+/* Selection rule (Sec. 3.3).  ENERGY_DRIFT: score_i = w_seg(i) * d_i with
+ * w = lambda + (1 - lambda) energy / max energy.  SEGMENT: the paper-literal
+ * anchor, d_i = 1 and lambda = 0 (whole loudest segments first).  DRIFT_ONLY:
+ * w = 1 (no audio guidance). */
+typedef enum {
+    ECHO_MODE_ENERGY_DRIFT = 0,
+    ECHO_MODE_SEGMENT = 1,
+    ECHO_MODE_DRIFT_ONLY = 2
+} echo_select_mode;
+
+typedef struct {
+    float lambda;   /* weight floor of silent segments, in [0, 1]; default 0.1 */
+    float xi;       /* Eq. 1 stabiliser, > 0; default 1e-6 */
+    int32_t mode;   /* echo_select_mode */
+} echo_select_params;
+
+typedef struct {
+    int32_t T;    /* latent frames = temporal segments */
+    int32_t N;    /* spatial latents per frame; NT = T * N tokens */
+    int32_t D;    /* hidden size, multiple of 64 */
+    int32_t H;    /* heads */
+    int32_t d;    /* head size, 64 or 128, H * d == D */
+    int32_t F;    /* FFN width, multiple of 64 */
+    int32_t Lc;   /* audio condition tokens, >= 1 */
+} echo_block_dims;
+
+/* Device pointers to one block's bf16 parameters, nn.Linear convention
+ * (y = x W^T + b, W row-major [out, in]).  Wkv stacks W_k over W_v ([2D, D]),
+ * bkv stacks b_k over b_v.  KVc is the block's cross-attention key|value
+ * table [Lc, 2D] (columns 0..D-1 keys, D..2D-1 values) from
+ * echo_precompute_cross_kv. */
+typedef struct {
+    const void *Wq, *bq;     /* [D, D], [D] */
+    const void *Wkv, *bkv;   /* [2D, D], [2D] */
+    const void *Wo, *bo;     /* [D, D], [D] */
+    const void *Wqc, *bqc;   /* [D, D], [D] */
+    const void *Woc, *boc;   /* [D, D], [D] */
+    const void *W1, *b1;     /* [F, D], [F] */
+    const void *W2, *b2;     /* [D, F], [D] */
+    const void *KVc;         /* [Lc, 2D] */
+} echo_block_weights;
+
+/* Human-readable name of a status.  Never NULL. */
+const char *echo_status_str(echo_status s);
+
+/* Synchronises `stream`, then reads and clears the device error flag shared by
+ * every kernel of this library on the current device.  Returns ECHO_OK, the
+ * flagged error (ECHO_ERR_NONFINITE, ECHO_ERR_TIMEOUT) or ECHO_ERR_CUDA if the
+ * synchronisation itself failed. */
+echo_status echo_get_device_error(echo_stream_t stream);
+
+/* Sec. 3.3 "Cross-modal Saliency Anchors": split the audio evenly into T
+ * segments, STFT each, energy = L2 norm of the segment's time-frequency matrix.
+ *   audio        f32 [n_samples], mono.  Segment length L_s = n_samples / T
+ *                (floor; the remainder is dropped).
+ *   n_fft        FFT size, power of two in [64, 4096]; hop >= 1; frames start
+ *                at 0, hop, ... while start + n_fft <= L_s (one zero-padded
+ *                frame if L_s < n_fft).  Periodic Hann window.
+ *   band_energy  f32 [T, n_bands] out: sum over frames of one-sided power
+ *                P_k = c_k |X_k|^2 / n_fft (c_0 = c_{n/2} = 1, else 2) over the
+ *                linear band [floor(B b / n_bands), floor(B (b+1) / n_bands)),
+ *                B = n_fft/2 + 1;  1 <= n_bands <= B.
+ *   seg_energy   f32 [T] out: sqrt(sum_b band_energy[tau, b]).
+ * Errors: INVALID_ARG (null/misaligned), SHAPE (T < 1, T > n_samples, bad
+ * n_fft/hop/n_bands), CUDA. */
+echo_status echo_audio_energy(const float *audio, int64_t n_samples, int32_t T,
+                              int32_t n_fft, int32_t hop, int32_t n_bands,
+                              float *band_energy, float *seg_energy,
+                              echo_stream_t stream);
+
+/* Bytes of workspace echo_select needs for NT = T * N tokens. */
+size_t echo_select_workspace_size(int32_t T, int32_t N);
+
+/* Sec. 3.3 (selection) with Eq. 1 applied per token against the cache.
+ *   x            [NT, D] layer input, dtype xt (ECHO_BF16 or ECHO_F32).
+ *   cache_q      int8 [NT, D], cache_scale f32 [NT]: the cached features
+ *                c_ij = float(q_ij) * s_i.
+ *   seg_energy   f32 [T] (echo_audio_energy output or any non-negative values).
+ *   ratio        refresh ratio ratio_num / ratio_den in [0, 1];
+ *                K = ceil(ratio_num * NT / ratio_den) computed in integers.
+ *   p            selection parameters (host pointer; NULL = defaults).
+ *   idx          int32 [>= K] out: the K active tokens, ascending.  The K
+ *                largest keys (score descending, index ascending) win.
+ *   K_out        host int32 out: K.
+ *   scores       f32 [NT] out (may be NULL): score_i = w_{i / N} * d_i with
+ *                d_i = sum_j |x_ij - c_ij| / (sum_j |c_ij| + xi), both sums
+ *                fp32 in a fixed order (8-element chunks left to right, chunk
+ *                c on lane c mod 32 in chunk order, then a xor butterfly
+ *                16, 8, 4, 2, 1), so that the result is reproducible bit for bit.
+ *   workspace    >= echo_select_workspace_size(T, N) bytes, 16-byte aligned.
+ * D must be a multiple of 8.  Errors: INVALID_ARG, SHAPE, WORKSPACE, CUDA;
+ * a non-finite score sets the NONFINITE device flag. */
+echo_status echo_select(const void *x, echo_dtype xt, const int8_t *cache_q,
+                        const float *cache_scale, const float *seg_energy,
+                        int32_t T, int32_t N, int32_t D, int32_t ratio_num,
+                        int32_t ratio_den, const echo_select_params *p,
+                        int32_t *idx, int32_t *K_out, float *scores,
+                        void *workspace, size_t ws_bytes, echo_stream_t stream);
+
+/* Bytes of workspace echo_block_step needs for dims and up to K_max active
+ * tokens (also enough for echo_precompute_cross_kv). */
+size_t echo_workspace_size(const echo_block_dims *dims, int32_t K_max);
+
+/* Cross-attention keys and values of the audio condition tokens, once per
+ * block and generation (the condition does not change across steps):
+ *   KVc[:, 0:D] = cond Wkc^T + bkc,  KVc[:, D:2D] = cond Wvc^T + bvc.
+ *   cond bf16 [Lc, D]; Wkvc bf16 [2D, D] (W_kc over W_vc); bkvc bf16 [2D];
+ *   KVc bf16 [Lc, 2D] out.  Errors: INVALID_ARG, SHAPE, CUDA. */
+echo_status echo_precompute_cross_kv(const void *cond, const void *Wkvc,
+                                     const void *bkvc, int32_t Lc, int32_t D,
+                                     void *KVc, echo_stream_t stream);
+
+/* Sec. 3.3 "Fine-grained latent-level caching" for one layer and one step:
+ *   n1 = LN(x) (all NT rows; LN: zero mean, unit variance, eps 1e-6, no affine)
+ *   K, V = n1 Wk^T + bk, n1 Wv^T + bv        (all latents)
+ *   Q'   = n1[idx] Wq^T + bq                  (active latents only)
+ *   h1   = x[idx] + MHA(Q', K, V) Wo^T + bo
+ *   h2   = h1 + MHA(LN(h1) Wqc^T + bqc, Kc, Vc) Woc^T + boc
+ *   y_act = h2 + GELU_tanh(LN(h2) W1^T + b1) W2^T + b2
+ *   cache[idx[j]] = int8 quantisation of bf16(y_act[j])   (Sec. 3.4)
+ *   y[i] = bf16(y_act[j]) if i == idx[j], else bf16(float(q_i) * s_i) from
+ *   the cache as it was on entry (mask fusion, Sec. 3.3).
+ *   x        bf16 [NT, D]; idx int32 [K] ascending, distinct, < NT (as from
+ *            echo_select); 0 <= K <= NT (K = 0 returns the reconstructed cache,
+ *            K = NT is the full step).
+ *   cache_q  int8 [NT, D], cache_scale f32 [NT], updated in place at idx.
+ *   y        bf16 [NT, D] out; may alias x.
+ *   workspace >= echo_workspace_size(dims, K) bytes, 256-byte aligned.
+ * Errors: INVALID_ARG, SHAPE, WORKSPACE, CUDA; NONFINITE/TIMEOUT device flags. */
+echo_status echo_block_step(const echo_block_weights *w, const echo_block_dims *dims,
+                            const void *x, const int32_t *idx, int32_t K,
+                            int8_t *cache_q, float *cache_scale, void *y,
+                            void *workspace, size_t ws_bytes, echo_stream_t stream);
+
+/* Sec. 3.4, int8 per-token symmetric quantisation:
+ *   q[rows[j]], scale[rows[j]] = Q(src[j]) for j < n_rows (rows NULL: j),
+ *   Q(v): a = max|v|; a == 0 -> s = 0, q = 0; else s = a / 127,
+ *   inv = 127 / a, q = clamp(round_half_even(v * inv), -127, 127), fp32.
+ *   src [n_rows, D] of dtype st; rows int32 [n_rows] distinct or NULL.
+ * D multiple of 8.  A non-finite amax writes q = 0, s = amax and sets the
+ * NONFINITE device flag.  Errors: INVALID_ARG, SHAPE, CUDA. */
+echo_status echo_cache_quant(const void *src, echo_dtype st, const int32_t *rows,
+                             int32_t n_rows, int32_t D, int8_t *q, float *scale,
+                             echo_stream_t stream);
+
+/* Sec. 3.4 reconstruction converted back to the compute precision:
+ *   dst[j] = cast(float(q[r]) * scale[r]), r = rows ? rows[j] : j, the product
+ *   in fp32 and the cast round-to-nearest-even (dt ECHO_BF16) or exact (ECHO_F32).
+ *   dst [n_rows, D].  D multiple of 16.  Errors: INVALID_ARG, SHAPE, CUDA. */
+echo_status echo_cache_dequant(const int8_t *q, const float *scale, const int32_t *rows,
+                               int32_t n_rows, int32_t D, void *dst, echo_dtype dt,
+                               echo_stream_t stream);
+
+/* ---- single kernels of echo_block_step, exported so that each can be
+ *      checked and timed on its own ---- */
+
+/* out = act(A W^T + bias) + resid: one tcgen05 bf16 GEMM (fp32 accumulate).
+ *   A bf16 [M, Kd] (row stride lda elements), W bf16 [N, Kd], bias bf16 [N]
+ *   or NULL; act 0 = none, 1 = GELU (tanh form).
+ *   resid: NULL, bf16 [*, N] read at row resid_rows[m] (or m if resid_rows is
+ *   NULL) when resid_t == ECHO_BF16, or f32 [M, N] when ECHO_F32.
+ *   out [M, N] (row stride ldo elements) of dtype out_t.
+ * Kd, N multiples of 64; lda, ldo multiples of 8.  Errors: INVALID_ARG, SHAPE, CUDA. */
+echo_status echo_linear(const void *A, int64_t lda, int32_t M, int32_t Kd,
+                        const void *W, const void *bias, int32_t N, int32_t act,
+                        const void *resid, echo_dtype resid_t, const int32_t *resid_rows,
+                        void *out, int64_t ldo, echo_dtype out_t, echo_stream_t stream);
+
+/* O[m, h d + e] = sum_j softmax_j(Q_h[m] . K_h[j] / sqrt(d)) V_h[j, e]:
+ *   Q bf16 [M, ldq], K and V bf16 [L, ldkv] (head h at columns h d .. h d + d - 1),
+ *   O bf16 [M, ldo].  d in {64, 128}; strides multiples of 8.
+ * Errors: INVALID_ARG, SHAPE, CUDA. */
+echo_status echo_attention(const void *Q, int64_t ldq, const void *K, const void *V,
+                           int64_t ldkv, int32_t M, int32_t L, int32_t H, int32_t d,
+                           void *O, int64_t ldo, echo_stream_t stream);
+
+/* out[j] = LN(in[rows ? rows[j] : j]) over D columns, eps 1e-6, no affine.
+ *   in [*, D] of dtype in_t, out bf16 [n_rows, D].  D multiple of 8.
+ * Errors: INVALID_ARG, SHAPE, CUDA. */
+echo_status echo_layernorm(const void *in, echo_dtype in_t, const int32_t *rows,
+                           int32_t n_rows, int32_t D, void *out, echo_stream_t stream);
+
+/* ---- instrumentation (no counterpart in the paper: measurement only) ---- */
+
+/* Kernel kinds reported by the profiler. */
+typedef enum {
+    ECHO_K_ENERGY = 0, ECHO_K_DRIFT = 1, ECHO_K_TOPK = 2, ECHO_K_ROWMAP = 3,
+    ECHO_K_LAYERNORM = 4, ECHO_K_GEMM = 5, ECHO_K_ATTENTION = 6, ECHO_K_QUANT = 7,
+    ECHO_K_DEQUANT = 8, ECHO_K_MERGE = 9, ECHO_K_COUNT = 10
+} echo_kernel_kind;
+
+/* Number of kernels this library has launched in this process (all devices). */
+uint64_t echo_launch_count(void);
+
+/* on != 0: from now on bracket every kernel launch with a pair of CUDA events
+ * recorded on the launch's own stream (up to 65536 launches are kept).
+ * on == 0: stop recording.  Recorded launches stay until read. */
+echo_status echo_profile_enable(int32_t on);
+
+/* Synchronises every recorded launch, copies up to `max` records (kind, the
+ * launch's shape m, n, k as described below, and its device time in ms) into
+ * the host arrays, clears the record list and returns the number copied (or
+ * -1 on a CUDA error).  Shapes: GEMM (M, N, Kd); ATTENTION (M queries, L keys,
+ * H * d); DRIFT (NT, D, 0); TOPK (NT, K, 0); LAYERNORM, QUANT, DEQUANT,
+ * MERGE (rows, D, 0); ENERGY (T, frames, n_fft). */
+int32_t echo_profile_read(int32_t max, int32_t *kinds, int64_t *m, int64_t *n, int64_t *k,
+                          float *ms);
+
+/* Name of a kernel kind ("gemm_tcgen05", ...).  Never NULL. */
+const char *echo_kernel_name(int32_t kind);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ECHOCACHE_H */

@@ -1,0 +1,138 @@
+// One cached layer step on the active latents (Sec. 3.3 "Fine-grained
+// latent-level caching", Sec. 3.4 for the cache write), as a fixed sequence of
+// stream-ordered kernels over a caller-owned workspace:
+//
+//   rowmap      token -> position in idx (or -1)
+//   LN          n1 = LN(x), all NT rows
+//   GEMM        KV = n1 [Wk; Wv]^T + [bk; bv]          (K, V over all latents)
+//   LN+gather   na = LN(x[idx])                         ("select active latents")
+//   GEMM        Q' = na Wq^T + bq
+//   attention   att = MHA(Q', K, V)
+//   GEMM        h1 = att Wo^T + bo + x[idx]             (fp32)
+//   LN, GEMM    Qc = LN(h1) Wqc^T + bqc
+//   attention   att = MHA(Qc, Kc, Vc)
+//   GEMM        h2 = att Woc^T + boc + h1               (fp32)
+//   LN, GEMM    u = GELU(LN(h2) W1^T + b1)
+//   GEMM        y_act = u W2^T + b2 + h2                (bf16)
+//   quant       cache[idx] = Q(y_act)
+//   merge       y = fresh rows at idx, reconstructed cache elsewhere
+#include "common.cuh"
+#include "internal.h"
+
+namespace {
+
+size_t al(size_t b) { return (b + 255) & ~(size_t)255; }
+
+struct Layout {
+    size_t rowmap, n1, kv, na, qa, att, h1, h2, u, yact, total;
+};
+
+Layout layout(const echo_block_dims &d, int64_t K) {
+    const int64_t NT = (int64_t)d.T * d.N;
+    Layout L;
+    size_t o = 0;
+    L.rowmap = o; o += al(sizeof(int32_t) * NT);
+    L.n1 = o;     o += al(2 * (size_t)NT * d.D);
+    L.kv = o;     o += al(2 * (size_t)NT * 2 * d.D);
+    L.na = o;     o += al(2 * (size_t)K * d.D);
+    L.qa = o;     o += al(2 * (size_t)K * d.D);
+    L.att = o;    o += al(2 * (size_t)K * d.D);
+    L.h1 = o;     o += al(4 * (size_t)K * d.D);
+    L.h2 = o;     o += al(4 * (size_t)K * d.D);
+    L.u = o;      o += al(2 * (size_t)K * d.F);
+    L.yact = o;   o += al(2 * (size_t)K * d.D);
+    L.total = o;
+    return L;
+}
+
+bool dims_ok(const echo_block_dims *d) {
+    if (!d) return false;
+    if (d->T < 1 || d->N < 1 || d->D < 64 || d->D % 64 || d->F < 64 || d->F % 64 || d->Lc < 1)
+        return false;
+    if ((d->d != 64 && d->d != 128) || d->H < 1 || (int64_t)d->H * d->d != d->D) return false;
+    if (d->D > 8192) return false;
+    if ((int64_t)d->T * d->N > (int64_t)INT32_MAX / 2) return false;
+    return true;
+}
+
+}  // namespace
+
+extern "C" size_t echo_workspace_size(const echo_block_dims *dims, int32_t K_max) {
+    if (!dims_ok(dims) || K_max < 0) return 0;
+    return layout(*dims, K_max).total;
+}
+
+extern "C" echo_status echo_precompute_cross_kv(const void *cond, const void *Wkvc,
+                                                const void *bkvc, int32_t Lc, int32_t D,
+                                                void *KVc, echo_stream_t stream) {
+    return echo_linear(cond, D, Lc, D, Wkvc, bkvc, 2 * D, 0, nullptr, ECHO_BF16, nullptr, KVc,
+                       2 * (int64_t)D, ECHO_BF16, stream);
+}
+
+extern "C" echo_status echo_block_step(const echo_block_weights *w, const echo_block_dims *dims,
+                                       const void *x, const int32_t *idx, int32_t K,
+                                       int8_t *cache_q, float *cache_scale, void *y,
+                                       void *workspace, size_t ws_bytes, echo_stream_t stream) {
+    using namespace echo;
+    if (!w || !dims || !x || !cache_q || !cache_scale || !y || !workspace) return ECHO_ERR_INVALID_ARG;
+    if (!dims_ok(dims)) return ECHO_ERR_SHAPE;
+    const echo_block_dims d = *dims;
+    const int NT = d.T * d.N;
+    if (K < 0 || K > NT) return ECHO_ERR_SHAPE;
+    if (K > 0 && !idx) return ECHO_ERR_INVALID_ARG;
+    const void *ptrs[] = {w->Wq, w->bq, w->Wkv, w->bkv, w->Wo, w->bo, w->Wqc, w->bqc,
+                          w->Woc, w->boc, w->W1, w->b1, w->W2, w->b2, w->KVc};
+    for (const void *p : ptrs)
+        if (!p || !aligned16(p)) return ECHO_ERR_INVALID_ARG;
+    if (!aligned16(x) || !aligned16(cache_q) || !aligned16(cache_scale) || !aligned16(y) ||
+        (idx && !aligned16(idx)) || (reinterpret_cast<uintptr_t>(workspace) & 255u))
+        return ECHO_ERR_INVALID_ARG;
+    const Layout L = layout(d, K);
+    if (ws_bytes < L.total) return ECHO_ERR_WORKSPACE;
+    if (!device_supported()) return ECHO_ERR_UNSUPPORTED;
+
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    int32_t *rowmap = reinterpret_cast<int32_t *>(ws + L.rowmap);
+    void *n1 = ws + L.n1, *kv = ws + L.kv, *na = ws + L.na, *qa = ws + L.qa, *att = ws + L.att;
+    void *h1 = ws + L.h1, *h2 = ws + L.h2, *u = ws + L.u, *yact = ws + L.yact;
+    const int D = d.D;
+    const __nv_bfloat16 *kvb = static_cast<const __nv_bfloat16 *>(kv);
+    const __nv_bfloat16 *kvc = static_cast<const __nv_bfloat16 *>(w->KVc);
+    echo_status s = ECHO_OK;
+
+    launch_rowmap(idx, K, NT, rowmap, st);
+    if (K > 0) {
+        launch_layernorm(x, ECHO_BF16, nullptr, NT, D, n1, st);
+        s = launch_linear({n1, D, NT, D, w->Wkv, w->bkv, 2 * D, 0, nullptr, ECHO_BF16, nullptr, kv,
+                           2 * (int64_t)D, ECHO_BF16}, st);
+        if (s != ECHO_OK) return s;
+        launch_layernorm(x, ECHO_BF16, idx, K, D, na, st);
+        s = launch_linear({na, D, K, D, w->Wq, w->bq, D, 0, nullptr, ECHO_BF16, nullptr, qa, D,
+                           ECHO_BF16}, st);
+        if (s != ECHO_OK) return s;
+        launch_attention(qa, D, kvb, kvb + D, 2 * (int64_t)D, K, NT, d.H, d.d, att, D, st);
+        s = launch_linear({att, D, K, D, w->Wo, w->bo, D, 0, x, ECHO_BF16, idx, h1, D, ECHO_F32}, st);
+        if (s != ECHO_OK) return s;
+        launch_layernorm(h1, ECHO_F32, nullptr, K, D, na, st);
+        s = launch_linear({na, D, K, D, w->Wqc, w->bqc, D, 0, nullptr, ECHO_BF16, nullptr, qa, D,
+                           ECHO_BF16}, st);
+        if (s != ECHO_OK) return s;
+        launch_attention(qa, D, kvc, kvc + D, 2 * (int64_t)D, K, d.Lc, d.H, d.d, att, D, st);
+        s = launch_linear({att, D, K, D, w->Woc, w->boc, D, 0, h1, ECHO_F32, nullptr, h2, D,
+                           ECHO_F32}, st);
+        if (s != ECHO_OK) return s;
+        launch_layernorm(h2, ECHO_F32, nullptr, K, D, na, st);
+        s = launch_linear({na, D, K, D, w->W1, w->b1, d.F, 1, nullptr, ECHO_BF16, nullptr, u, d.F,
+                           ECHO_BF16}, st);
+        if (s != ECHO_OK) return s;
+        s = launch_linear({u, d.F, K, d.F, w->W2, w->b2, D, 0, h2, ECHO_F32, nullptr, yact, D,
+                           ECHO_BF16}, st);
+        if (s != ECHO_OK) return s;
+    }
+    // the merge reads the cache of the inactive rows only, the quantiser writes
+    // the active rows only: their order does not matter
+    launch_dequant_merge(cache_q, cache_scale, rowmap, yact, NT, D, y, st);
+    if (K > 0) launch_quant(yact, ECHO_BF16, idx, K, D, cache_q, cache_scale, st);
+    return last_launch_status();
+}

@@ -1,0 +1,280 @@
+// Dense bf16 projections of the block (Q', K/V over all latents, output
+// projections, FFN on the active latents; Sec. 3.3) on the 5th-generation
+// tensor cores:  out = act(A W^T + bias) + resid.
+//
+// One CTA per 128 x 256 output tile, 8 warps:
+//   warp 0      TMA producer: A [128 x 64] and W [256 x 64] bf16 tiles, 128-byte
+//               swizzle, into a 4-stage shared-memory ring (48 KB per stage);
+//   warp 1      one elected thread issues tcgen05.mma (M=128, N=256, K=16) into a
+//               128 x 256 fp32 accumulator in tensor memory, and commits each
+//               stage back to the producer;
+//   warp 2      allocates / frees the 256 tensor-memory columns;
+//   warps 4..7  epilogue: tcgen05.ld 32 columns at a time (warp w reads TMEM
+//               lanes 32 (w mod 4) ..), adds bias, GELU, residual, stores.
+// Every mbarrier wait is bounded (ECHO_ERR_TIMEOUT) and a CTA that gives up
+// drains its own copies and MMAs before it frees tensor memory.
+#include "common.cuh"
+#include "internal.h"
+
+namespace {
+
+constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2;   // 16 KB
+constexpr int B_BYTES = BN * BK * 2;   // 32 KB
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024;  // + alignment slack
+constexpr int THREADS = 256;
+constexpr uint32_t TMEM_COLS = 256;
+constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
+
+enum : int { EPI_GELU = 1, EPI_RES_BF16 = 2, EPI_RES_F32 = 4, EPI_OUT_F32 = 8 };
+
+struct GemmParams {
+    int M, N, Kd;
+    const __nv_bfloat16 *bias;
+    const void *resid;
+    const int32_t *resid_rows;
+    void *out;
+    int64_t ldo;
+    int *err;
+};
+
+ECHO_DEV float gelu_tanh(float x) {
+    const float k0 = 0.7978845608028654f;  // sqrt(2 / pi)
+    const float u = k0 * (x + 0.044715f * x * x * x);
+    return 0.5f * x * (1.f + tanhf(u));
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(THREADS, 1)
+gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+            const GemmParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                ~static_cast<uintptr_t>(1023));
+    __shared__ __align__(8) uint64_t full_bar[STAGES], empty_bar[STAGES], accum_bar, drain_bar;
+    __shared__ uint32_t tmem_slot;
+    __shared__ int abort_flag;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM;
+    const int num_kb = p.Kd / BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(&full_bar[s], 1);
+            mbar_init(&empty_bar[s], 1);
+        }
+        mbar_init(&accum_bar, 1);
+        mbar_init(&drain_bar, 1);
+        abort_flag = 0;
+        fence_barrier_init();
+        tma_prefetch_desc(&tmA);
+        tma_prefetch_desc(&tmB);
+    }
+    if (warp == 2) tmem_alloc(&tmem_slot, TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+    volatile int *abort_v = &abort_flag;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer ----------------
+        int issued = 0;
+        for (int kb = 0; kb < num_kb; ++kb) {
+            const int s = kb % STAGES;
+            const uint32_t ph = (kb / STAGES) & 1;
+            if (!mbar_wait(&empty_bar[s], ph ^ 1, abort_v, p.err)) break;
+            uint8_t *a = smem + s * STAGE_BYTES;
+            uint8_t *b = a + A_BYTES;
+            mbar_arrive_expect_tx(&full_bar[s], STAGE_BYTES);
+            tma_load_2d(a, &tmA, &full_bar[s], kb * BK, m0);
+            tma_load_2d(b, &tmB, &full_bar[s], kb * BK, n0);
+            issued = kb + 1;
+        }
+        if (*abort_v) {  // let this CTA's copies land before it exits
+            for (int kb = issued - STAGES < 0 ? 0 : issued - STAGES; kb < issued; ++kb)
+                mbar_wait(&full_bar[kb % STAGES], (kb / STAGES) & 1, abort_v, nullptr, 100000000ull);
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer ----------------
+        bool ok = true;
+        for (int kb = 0; kb < num_kb; ++kb) {
+            const int s = kb % STAGES;
+            const uint32_t ph = (kb / STAGES) & 1;
+            if (!mbar_wait(&full_bar[s], ph, abort_v, p.err)) { ok = false; break; }
+            tc_fence_after();
+            const uint8_t *a = smem + s * STAGE_BYTES;
+            const uint8_t *b = a + A_BYTES;
+#pragma unroll
+            for (int k = 0; k < BK / 16; ++k) {
+                const uint64_t ad = smem_desc_sw128(a + k * 32);
+                const uint64_t bd = smem_desc_sw128(b + k * 32);
+                tc_mma_f16(tmem, ad, bd, IDESC, (kb | k) != 0);
+            }
+            tc_commit(&empty_bar[s]);
+        }
+        if (ok) {
+            tc_commit(&accum_bar);
+        } else {  // wait for the MMAs already issued before tensor memory is freed
+            tc_commit(&drain_bar);
+            mbar_wait(&drain_bar, 0, abort_v, nullptr, 100000000ull);
+        }
+    } else if (warp >= 4) {
+        // ---------------- epilogue ----------------
+        const int q = warp & 3;
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(&accum_bar, 0, abort_v, p.err,
+                                                          4000000000ull));
+        tc_fence_after();
+        if (ok) {
+            const int row = m0 + q * 32 + lane;
+            const bool row_ok = row < p.M;
+            int rrow = row;
+            if ((EPI & EPI_RES_BF16) && p.resid_rows && row_ok) rrow = p.resid_rows[row];
+            for (int c = 0; c < BN; c += 32) {
+                const int col = n0 + c;
+                if (col >= p.N) break;                       // warp-uniform
+                uint32_t r[32];
+                tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c, r);
+                tmem_ld_wait();
+                if (!row_ok) continue;
+                float v[32];
+                if (p.bias) {
+                    const uint4 *bp = reinterpret_cast<const uint4 *>(p.bias + col);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) unpack8_bf16(__ldg(bp + i), v + 8 * i);
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] += __uint_as_float(r[i]);
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+                }
+                if (EPI & EPI_GELU) {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = gelu_tanh(v[i]);
+                }
+                if (EPI & EPI_RES_BF16) {
+                    const uint4 *rp = reinterpret_cast<const uint4 *>(
+                        static_cast<const __nv_bfloat16 *>(p.resid) + (int64_t)rrow * p.N + col);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        float t[8];
+                        unpack8_bf16(__ldg(rp + i), t);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) v[8 * i + e] += t[e];
+                    }
+                }
+                if (EPI & EPI_RES_F32) {
+                    const float4 *rp = reinterpret_cast<const float4 *>(
+                        static_cast<const float *>(p.resid) + (int64_t)row * p.N + col);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const float4 t = __ldg(rp + i);
+                        v[4 * i] += t.x; v[4 * i + 1] += t.y; v[4 * i + 2] += t.z; v[4 * i + 3] += t.w;
+                    }
+                }
+                if (EPI & EPI_OUT_F32) {
+                    float4 *op = reinterpret_cast<float4 *>(static_cast<float *>(p.out) +
+                                                            (int64_t)row * p.ldo + col);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        op[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+                } else {
+                    uint4 *op = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.out) +
+                                                          (int64_t)row * p.ldo + col);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) op[i] = pack8_bf16(v + 8 * i);
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 2) {
+        tc_fence_after();
+        tmem_dealloc(tmem, TMEM_COLS);
+    }
+}
+
+template <int EPI>
+echo_status run(const CUtensorMap &ta, const CUtensorMap &tb, const GemmParams &p, cudaStream_t st) {
+    static int attr_set[64] = {};  // per device; a benign race sets the same value twice
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return ECHO_ERR_CUDA;
+    if (!attr_set[dev]) {
+        if (cudaFuncSetAttribute(gemm_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 SMEM_BYTES) != cudaSuccess)
+            return ECHO_ERR_CUDA;
+        attr_set[dev] = 1;
+    }
+    dim3 grid((p.N + BN - 1) / BN, (p.M + BM - 1) / BM);
+    echo::LaunchScope ls(ECHO_K_GEMM, p.M, p.N, p.Kd, st);
+    gemm_kernel<EPI><<<grid, THREADS, SMEM_BYTES, st>>>(ta, tb, p);
+    return echo::last_launch_status();
+}
+
+}  // namespace
+
+namespace echo {
+
+echo_status launch_linear(const LinearArgs &a, cudaStream_t st) {
+    if (a.M <= 0) return ECHO_OK;
+    CUtensorMap ta, tb;
+    if (!make_tmap_bf16(&ta, a.A, (uint64_t)a.M, (uint64_t)a.Kd, (uint64_t)a.lda, BM) ||
+        !make_tmap_bf16(&tb, a.W, (uint64_t)a.N, (uint64_t)a.Kd, (uint64_t)a.Kd, BN))
+        return ECHO_ERR_CUDA;
+    GemmParams p;
+    p.M = a.M; p.N = a.N; p.Kd = a.Kd;
+    p.bias = static_cast<const __nv_bfloat16 *>(a.bias);
+    p.resid = a.resid;
+    p.resid_rows = a.resid_rows;
+    p.out = a.out;
+    p.ldo = a.ldo;
+    p.err = device_error_ptr();
+    int epi = 0;
+    if (a.act == 1) epi |= EPI_GELU;
+    if (a.resid) epi |= (a.resid_t == ECHO_BF16) ? EPI_RES_BF16 : EPI_RES_F32;
+    if (a.out_t == ECHO_F32) epi |= EPI_OUT_F32;
+    switch (epi) {
+        case 0: return run<0>(ta, tb, p, st);
+        case EPI_GELU: return run<EPI_GELU>(ta, tb, p, st);
+        case EPI_RES_BF16: return run<EPI_RES_BF16>(ta, tb, p, st);
+        case EPI_RES_F32: return run<EPI_RES_F32>(ta, tb, p, st);
+        case EPI_GELU | EPI_RES_BF16: return run<EPI_GELU | EPI_RES_BF16>(ta, tb, p, st);
+        case EPI_GELU | EPI_RES_F32: return run<EPI_GELU | EPI_RES_F32>(ta, tb, p, st);
+        case EPI_OUT_F32: return run<EPI_OUT_F32>(ta, tb, p, st);
+        case EPI_GELU | EPI_OUT_F32: return run<EPI_GELU | EPI_OUT_F32>(ta, tb, p, st);
+        case EPI_RES_BF16 | EPI_OUT_F32: return run<EPI_RES_BF16 | EPI_OUT_F32>(ta, tb, p, st);
+        case EPI_RES_F32 | EPI_OUT_F32: return run<EPI_RES_F32 | EPI_OUT_F32>(ta, tb, p, st);
+        case EPI_GELU | EPI_RES_BF16 | EPI_OUT_F32:
+            return run<EPI_GELU | EPI_RES_BF16 | EPI_OUT_F32>(ta, tb, p, st);
+        case EPI_GELU | EPI_RES_F32 | EPI_OUT_F32:
+            return run<EPI_GELU | EPI_RES_F32 | EPI_OUT_F32>(ta, tb, p, st);
+    }
+    return ECHO_ERR_INVALID_ARG;
+}
+
+}  // namespace echo
+
+extern "C" echo_status echo_linear(const void *A, int64_t lda, int32_t M, int32_t Kd, const void *W,
+                                   const void *bias, int32_t N, int32_t act, const void *resid,
+                                   echo_dtype resid_t, const int32_t *resid_rows, void *out,
+                                   int64_t ldo, echo_dtype out_t, echo_stream_t stream) {
+    using namespace echo;
+    if (M < 0 || Kd < 64 || Kd % 64 || N < 64 || N % 64) return ECHO_ERR_SHAPE;
+    if (lda < Kd || lda % 8 || ldo < N || ldo % 8) return ECHO_ERR_SHAPE;
+    if (M == 0) return ECHO_OK;
+    if (!A || !W || !out) return ECHO_ERR_INVALID_ARG;
+    if (act != 0 && act != 1) return ECHO_ERR_INVALID_ARG;
+    if ((resid && resid_t != ECHO_BF16 && resid_t != ECHO_F32) ||
+        (out_t != ECHO_BF16 && out_t != ECHO_F32))
+        return ECHO_ERR_INVALID_ARG;
+    if (resid_rows && (!resid || resid_t != ECHO_BF16)) return ECHO_ERR_INVALID_ARG;
+    if (!aligned16(A) || !aligned16(W) || !aligned16(out) || (bias && !aligned16(bias)) ||
+        (resid && !aligned16(resid)) || (resid_rows && !aligned16(resid_rows)))
+        return ECHO_ERR_INVALID_ARG;
+    if (!device_supported()) return ECHO_ERR_UNSUPPORTED;
+    LinearArgs a{A, lda, M, Kd, W, bias, N, act, resid, resid_t, resid_rows, out, ldo, out_t};
+    return launch_linear(a, reinterpret_cast<cudaStream_t>(stream));
+}

@@ -1,0 +1,151 @@
+// Layer norm without affine, eps 1e-6, biased variance (the block's LN), with
+// an optional row gather: out[j] = LN(in[rows[j]]).  The gathered form is the
+// "select active latents" step of Sec. 3.3 fused with the LN that follows it.
+//
+// A row lives in registers (up to 8 chunks of 8 values per thread): one warp
+// per row for D <= 1024, four warps per row up to D = 8192.  Mean first, then
+// the centred variance, both fp32 tree reductions; one HBM read, one write.
+#include "common.cuh"
+#include "internal.h"
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kMaxChunks = 8;
+
+template <typename T>
+ECHO_DEV void ld8(const T *p, float *f);
+template <>
+ECHO_DEV void ld8<__nv_bfloat16>(const __nv_bfloat16 *p, float *f) {
+    unpack8_bf16(__ldg(reinterpret_cast<const uint4 *>(p)), f);
+}
+template <>
+ECHO_DEV void ld8<float>(const float *p, float *f) {
+    const float4 a = __ldg(reinterpret_cast<const float4 *>(p));
+    const float4 b = __ldg(reinterpret_cast<const float4 *>(p) + 1);
+    f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w;
+    f[4] = b.x; f[5] = b.y; f[6] = b.z; f[7] = b.w;
+}
+
+template <int TPR>
+ECHO_DEV float row_sum(float v, float *red) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if (TPR == 32) return v;
+    constexpr int W = TPR / 32;
+    const int warp = threadIdx.x >> 5;
+    const int row_in_block = threadIdx.x / TPR;
+    __syncthreads();
+    if ((threadIdx.x & 31) == 0) red[warp] = v;
+    __syncthreads();
+    float s = 0.f;
+#pragma unroll
+    for (int w = 0; w < W; ++w) s += red[row_in_block * W + w];
+    return s;
+}
+
+template <typename T, int TPR>
+__global__ void __launch_bounds__(kThreads)
+layernorm_kernel(const T *__restrict__ in, const int32_t *__restrict__ rows, int n_rows, int D,
+                 __nv_bfloat16 *__restrict__ out) {
+    __shared__ float red[kThreads / 32];
+    constexpr int RPB = kThreads / TPR;
+    const int t = threadIdx.x % TPR;
+    const int C = D >> 3;
+    const float invD = 1.f / (float)D;
+    for (int base = blockIdx.x * RPB; base < n_rows; base += gridDim.x * RPB) {
+        const int j = base + threadIdx.x / TPR;
+        const bool live = j < n_rows;
+        const int r = live ? (rows ? rows[j] : j) : 0;
+        const T *src = in + (int64_t)r * D;
+        float v[kMaxChunks][8];
+        float s = 0.f;
+#pragma unroll
+        for (int k = 0; k < kMaxChunks; ++k) {
+            const int c = t + k * TPR;
+            if (live && c < C) {
+                ld8<T>(src + 8 * c, v[k]);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) s += v[k][e];
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) v[k][e] = 0.f;
+            }
+        }
+        const float mean = row_sum<TPR>(s, red) * invD;
+        float ss = 0.f;
+#pragma unroll
+        for (int k = 0; k < kMaxChunks; ++k) {
+            const int c = t + k * TPR;
+            if (live && c < C) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const float dlt = v[k][e] - mean;
+                    ss += dlt * dlt;
+                }
+            }
+        }
+        const float var = row_sum<TPR>(ss, red) * invD;
+        const float rstd = rsqrtf(var + 1e-6f);
+        if (live) {
+            __nv_bfloat16 *dst = out + (int64_t)j * D;
+#pragma unroll
+            for (int k = 0; k < kMaxChunks; ++k) {
+                const int c = t + k * TPR;
+                if (c < C) {
+                    float o[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) o[e] = (v[k][e] - mean) * rstd;
+                    *reinterpret_cast<uint4 *>(dst + 8 * c) = pack8_bf16(o);
+                }
+            }
+        }
+    }
+}
+
+template <typename T>
+void launch_t(const T *in, const int32_t *rows, int n_rows, int D, __nv_bfloat16 *out,
+              cudaStream_t st) {
+    const int C = D / 8;
+    echo::LaunchScope ls(ECHO_K_LAYERNORM, n_rows, D, 0, st);
+    if (C <= 32 * kMaxChunks / 2) {   // D <= 1024: a warp per row
+        constexpr int RPB = kThreads / 32;
+        int grid = (n_rows + RPB - 1) / RPB;
+        if (grid > 152 * 16) grid = 152 * 16;
+        layernorm_kernel<T, 32><<<grid, kThreads, 0, st>>>(in, rows, n_rows, D, out);
+    } else {
+        constexpr int RPB = kThreads / 128;
+        int grid = (n_rows + RPB - 1) / RPB;
+        if (grid > 152 * 16) grid = 152 * 16;
+        layernorm_kernel<T, 128><<<grid, kThreads, 0, st>>>(in, rows, n_rows, D, out);
+    }
+}
+
+}  // namespace
+
+namespace echo {
+
+void launch_layernorm(const void *in, echo_dtype in_t, const int32_t *rows, int32_t n_rows,
+                      int32_t D, void *out, cudaStream_t st) {
+    if (n_rows <= 0) return;
+    __nv_bfloat16 *o = static_cast<__nv_bfloat16 *>(out);
+    if (in_t == ECHO_BF16)
+        launch_t(static_cast<const __nv_bfloat16 *>(in), rows, n_rows, D, o, st);
+    else
+        launch_t(static_cast<const float *>(in), rows, n_rows, D, o, st);
+}
+
+}  // namespace echo
+
+extern "C" echo_status echo_layernorm(const void *in, echo_dtype in_t, const int32_t *rows,
+                                      int32_t n_rows, int32_t D, void *out, echo_stream_t stream) {
+    using namespace echo;
+    if (n_rows < 0 || D < 8 || D % 8 || D > 8192) return ECHO_ERR_SHAPE;
+    if (n_rows == 0) return ECHO_OK;
+    if (!in || !out) return ECHO_ERR_INVALID_ARG;
+    if (in_t != ECHO_BF16 && in_t != ECHO_F32) return ECHO_ERR_INVALID_ARG;
+    if (!aligned16(in) || !aligned16(out) || (rows && !aligned16(rows))) return ECHO_ERR_INVALID_ARG;
+    if (!device_supported()) return ECHO_ERR_UNSUPPORTED;
+    launch_layernorm(in, in_t, rows, n_rows, D, out, reinterpret_cast<cudaStream_t>(stream));
+    return last_launch_status();
+}

@@ -1,0 +1,337 @@
+// Token selection (Sec. 3.3): per-token drift (Eq. 1 applied per token against
+// the int8 cache), weighted by the token's segment energy, then top-K by
+// (score descending, index ascending) returned as an ascending index list.
+//
+// drift_kernel: one warp per token row, 128-bit loads of x and 64-bit loads of
+//   the int8 cache; the two L1 sums are fp32 in the canonical order (lane l owns
+//   8-element chunks l, l+32, ...; chunk sums left to right; xor butterfly
+//   16..1), with explicit round-to-nearest intrinsics so nothing is contracted.
+// topk_kernel: one CTA radix-selects the K-th largest 32-bit key (11/11/10-bit
+//   digits), then compacts in index order, taking keys equal to the threshold
+//   from the lowest index up.
+#include "common.cuh"
+#include "internal.h"
+
+namespace {
+
+constexpr int kDriftThreads = 256;
+constexpr int kDriftUnroll = 4;
+constexpr int kTopkThreads = 1024;
+constexpr int kTopkItems = 4;
+
+ECHO_DEV float segment_weight(float e, float emax, float lam) {
+    if (!(emax > 0.f)) return 1.f;
+    const float t = __fdiv_rn(e, emax);
+    return __fadd_rn(lam, __fmul_rn(__fsub_rn(1.f, lam), t));
+}
+
+template <typename XT>
+struct XChunk;
+
+template <>
+struct XChunk<__nv_bfloat16> {
+    uint4 v;
+    ECHO_DEV void load(const __nv_bfloat16 *p) { v = __ldcs(reinterpret_cast<const uint4 *>(p)); }
+    ECHO_DEV void get(float *f) const { unpack8_bf16(v, f); }
+};
+
+template <>
+struct XChunk<float> {
+    float4 a, b;
+    ECHO_DEV void load(const float *p) {
+        a = __ldcs(reinterpret_cast<const float4 *>(p));
+        b = __ldcs(reinterpret_cast<const float4 *>(p) + 1);
+    }
+    ECHO_DEV void get(float *f) const {
+        f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w;
+        f[4] = b.x; f[5] = b.y; f[6] = b.z; f[7] = b.w;
+    }
+};
+
+template <typename XT>
+__global__ void __launch_bounds__(kDriftThreads)
+drift_kernel(const XT *__restrict__ x, const int8_t *__restrict__ q, const float *__restrict__ scale,
+             const float *__restrict__ seg_energy, int T, int N, int NT, int D, float lam, float xi,
+             int mode, float *__restrict__ scores, int *err) {
+    __shared__ float s_emax;
+    if (threadIdx.x < 32) {
+        float m = 0.f;
+        for (int i = threadIdx.x; i < T; i += 32) m = fmaxf(m, seg_energy[i]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+        if (threadIdx.x == 0) s_emax = m;
+    }
+    __syncthreads();
+    const float emax = s_emax;
+    const int lane = threadIdx.x & 31;
+    const int warps = blockDim.x >> 5;
+    const int C = D >> 3;
+    for (int row = blockIdx.x * warps + (threadIdx.x >> 5); row < NT; row += gridDim.x * warps) {
+        const int seg = row / N;
+        const float e = seg_energy[seg];
+        float w;
+        if (mode == ECHO_MODE_SEGMENT) w = segment_weight(e, emax, 0.f);
+        else if (mode == ECHO_MODE_DRIFT_ONLY) w = 1.f;
+        else w = segment_weight(e, emax, lam);
+
+        float d = 1.f;
+        if (mode != ECHO_MODE_SEGMENT) {
+            const float sc = scale[row];
+            const XT *xr = x + (int64_t)row * D;
+            const int8_t *qr = q + (int64_t)row * D;
+            float num = 0.f, den = 0.f;
+            for (int c0 = lane; c0 < C; c0 += 32 * kDriftUnroll) {
+                XChunk<XT> xv[kDriftUnroll];
+                uint2 qv[kDriftUnroll];
+#pragma unroll
+                for (int u = 0; u < kDriftUnroll; ++u) {
+                    const int c = c0 + 32 * u;
+                    if (c < C) {
+                        xv[u].load(xr + 8 * c);
+                        qv[u] = __ldcs(reinterpret_cast<const uint2 *>(qr + 8 * c));
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < kDriftUnroll; ++u) {
+                    const int c = c0 + 32 * u;
+                    if (c < C) {
+                        float xf[8];
+                        xv[u].get(xf);
+                        const int8_t *qb = reinterpret_cast<const int8_t *>(&qv[u]);
+                        float cn = 0.f, cd = 0.f;
+#pragma unroll
+                        for (int k = 0; k < 8; ++k) {
+                            const float ch = __fmul_rn((float)qb[k], sc);
+                            const float an = fabsf(__fsub_rn(xf[k], ch));
+                            const float ad = fabsf(ch);
+                            cn = k ? __fadd_rn(cn, an) : an;
+                            cd = k ? __fadd_rn(cd, ad) : ad;
+                        }
+                        num = __fadd_rn(num, cn);
+                        den = __fadd_rn(den, cd);
+                    }
+                }
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                num = __fadd_rn(num, __shfl_xor_sync(0xffffffffu, num, o));
+                den = __fadd_rn(den, __shfl_xor_sync(0xffffffffu, den, o));
+            }
+            d = __fdiv_rn(num, __fadd_rn(den, xi));
+        }
+        const float score = __fmul_rn(w, d);
+        if (lane == 0) {
+            scores[row] = score;
+            if (!isfinite(score)) echo_flag_error(err, ECHO_ERR_NONFINITE);
+        }
+    }
+}
+
+ECHO_DEV uint32_t order_key(float f) {
+    const uint32_t b = __float_as_uint(f);
+    return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+// Exclusive block scan of one value per thread (blockDim == kTopkThreads).
+// Returns the exclusive prefix; *total gets the block sum.
+ECHO_DEV int block_exclusive_scan(int v, int *warp_sums, int *total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int inc = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int n = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += n;
+    }
+    if (lane == 31) warp_sums[warp] = inc;
+    __syncthreads();
+    if (warp == 0) {
+        int w = warp_sums[lane];
+        int wi = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int n = __shfl_up_sync(0xffffffffu, wi, o);
+            if (lane >= o) wi += n;
+        }
+        warp_sums[lane] = wi - w;           // exclusive prefix of warp totals
+        if (lane == 31) warp_sums[32] = wi; // block total
+    }
+    __syncthreads();
+    const int r = warp_sums[warp] + inc - v;
+    *total = warp_sums[32];
+    __syncthreads();
+    return r;
+}
+
+__global__ void __launch_bounds__(kTopkThreads)
+topk_kernel(const float *__restrict__ scores, int NT, int K, int keys_in_smem,
+            int32_t *__restrict__ idx) {
+    extern __shared__ uint32_t skeys[];
+    __shared__ int hist[2048];
+    __shared__ int warp_sums[33];
+    __shared__ int s_digit, s_krem;
+    const int tid = threadIdx.x;
+
+    if (K >= NT) {
+        for (int i = tid; i < NT; i += blockDim.x) idx[i] = i;
+        return;
+    }
+    if (K <= 0) return;
+
+    if (keys_in_smem)
+        for (int i = tid; i < NT; i += blockDim.x) skeys[i] = order_key(scores[i]);
+    __syncthreads();
+    auto key_at = [&](int i) -> uint32_t {
+        return keys_in_smem ? skeys[i] : order_key(scores[i]);
+    };
+
+    uint32_t prefix = 0, pmask = 0;
+    int krem = K;
+    const int shifts[3] = {21, 10, 0};
+    const int widths[3] = {11, 11, 10};
+    for (int pass = 0; pass < 3; ++pass) {
+        const int sh = shifts[pass];
+        const int nb = 1 << widths[pass];
+        for (int b = tid; b < 2048; b += blockDim.x) hist[b] = 0;
+        __syncthreads();
+        for (int i = tid; i < NT; i += blockDim.x) {
+            const uint32_t k = key_at(i);
+            if ((k & pmask) == prefix) atomicAdd(&hist[(k >> sh) & (nb - 1)], 1);
+        }
+        __syncthreads();
+        // thread t covers the two bins hi = nb-1-2t and lo = hi-1 (descending)
+        const int hi = nb - 1 - 2 * tid;
+        int c_hi = 0, c_lo = 0;
+        if (hi >= 0) c_hi = hist[hi];
+        if (hi - 1 >= 0) c_lo = hist[hi - 1];
+        int total;
+        const int above = block_exclusive_scan(c_hi + c_lo, warp_sums, &total);
+        if (hi >= 0 && above < krem && above + c_hi >= krem) {
+            s_digit = hi;
+            s_krem = krem - above;
+        }
+        if (hi - 1 >= 0 && above + c_hi < krem && above + c_hi + c_lo >= krem) {
+            s_digit = hi - 1;
+            s_krem = krem - above - c_hi;
+        }
+        __syncthreads();
+        prefix |= (uint32_t)s_digit << sh;
+        pmask |= (uint32_t)(nb - 1) << sh;
+        krem = s_krem;
+        __syncthreads();
+    }
+    // prefix is the K-th largest key; take every larger key and the first
+    // `krem` keys equal to it in index order.
+    const uint32_t thr = prefix;
+    const int need_eq = krem;
+    int eq_run = 0, sel_run = 0;
+    const int tile = kTopkThreads * kTopkItems;
+    for (int base = 0; base < NT; base += tile) {
+        bool gt[kTopkItems], eq[kTopkItems];
+        int neq = 0;
+#pragma unroll
+        for (int j = 0; j < kTopkItems; ++j) {
+            const int i = base + tid * kTopkItems + j;
+            gt[j] = eq[j] = false;
+            if (i < NT) {
+                const uint32_t k = key_at(i);
+                gt[j] = k > thr;
+                eq[j] = k == thr;
+            }
+            neq += eq[j];
+        }
+        int eq_total;
+        int eq_before = eq_run + block_exclusive_scan(neq, warp_sums, &eq_total);
+        bool sel[kTopkItems];
+        int nsel = 0;
+#pragma unroll
+        for (int j = 0; j < kTopkItems; ++j) {
+            sel[j] = gt[j];
+            if (eq[j]) {
+                sel[j] = eq_before < need_eq;
+                ++eq_before;
+            }
+            nsel += sel[j];
+        }
+        int sel_total;
+        int pos = sel_run + block_exclusive_scan(nsel, warp_sums, &sel_total);
+#pragma unroll
+        for (int j = 0; j < kTopkItems; ++j)
+            if (sel[j]) idx[pos++] = base + tid * kTopkItems + j;
+        eq_run += eq_total;
+        sel_run += sel_total;
+    }
+}
+
+size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
+
+}  // namespace
+
+extern "C" size_t echo_select_workspace_size(int32_t T, int32_t N) {
+    if (T < 1 || N < 1) return 0;
+    return align256((size_t)T * N * sizeof(float));
+}
+
+extern "C" echo_status echo_select(const void *x, echo_dtype xt, const int8_t *cache_q,
+                                   const float *cache_scale, const float *seg_energy, int32_t T,
+                                   int32_t N, int32_t D, int32_t ratio_num, int32_t ratio_den,
+                                   const echo_select_params *p, int32_t *idx, int32_t *K_out,
+                                   float *scores, void *workspace, size_t ws_bytes,
+                                   echo_stream_t stream) {
+    using namespace echo;
+    if (!x || !cache_q || !cache_scale || !seg_energy || !idx || !K_out) return ECHO_ERR_INVALID_ARG;
+    if (xt != ECHO_BF16 && xt != ECHO_F32) return ECHO_ERR_INVALID_ARG;
+    if (!aligned16(x) || !aligned16(cache_q) || !aligned16(cache_scale) || !aligned16(seg_energy) ||
+        !aligned16(idx) || (scores && !aligned16(scores)))
+        return ECHO_ERR_INVALID_ARG;
+    echo_select_params prm = {0.1f, 1e-6f, ECHO_MODE_ENERGY_DRIFT};
+    if (p) prm = *p;
+    if (prm.mode < 0 || prm.mode > 2 || !(prm.xi > 0.f) || !(prm.lambda >= 0.f) ||
+        !(prm.lambda <= 1.f))
+        return ECHO_ERR_INVALID_ARG;
+    if (T < 1 || N < 1 || D < 8 || D % 8 || ratio_den < 1 || ratio_num < 0 || ratio_num > ratio_den)
+        return ECHO_ERR_SHAPE;
+    const int64_t NT64 = (int64_t)T * N;
+    if (NT64 > (int64_t)INT32_MAX / 2) return ECHO_ERR_SHAPE;
+    const int NT = (int)NT64;
+    const int K = (int)(((int64_t)ratio_num * NT + ratio_den - 1) / ratio_den);
+    float *sc = scores;
+    if (!sc) {
+        if (!workspace || !aligned16(workspace)) return ECHO_ERR_INVALID_ARG;
+        if (ws_bytes < echo_select_workspace_size(T, N)) return ECHO_ERR_WORKSPACE;
+        sc = static_cast<float *>(workspace);
+    }
+    if (!device_supported()) return ECHO_ERR_UNSUPPORTED;
+    *K_out = K;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    int *err = device_error_ptr();
+
+    const int warps = kDriftThreads / 32;
+    int grid = (NT + warps - 1) / warps;
+    {
+    LaunchScope ls(ECHO_K_DRIFT, NT, D, 0, st);
+    if (xt == ECHO_BF16)
+        drift_kernel<__nv_bfloat16><<<grid, kDriftThreads, 0, st>>>(
+            static_cast<const __nv_bfloat16 *>(x), cache_q, cache_scale, seg_energy, T, N, NT, D,
+            prm.lambda, prm.xi, prm.mode, sc, err);
+    else
+        drift_kernel<float><<<grid, kDriftThreads, 0, st>>>(
+            static_cast<const float *>(x), cache_q, cache_scale, seg_energy, T, N, NT, D,
+            prm.lambda, prm.xi, prm.mode, sc, err);
+    }
+    if (last_launch_status() != ECHO_OK) return ECHO_ERR_CUDA;
+
+    // keys staged in shared memory when they fit next to the static buffers
+    const size_t key_bytes = (size_t)NT * sizeof(uint32_t);
+    const size_t max_dyn = 200 * 1024;
+    const int in_smem = key_bytes <= max_dyn ? 1 : 0;
+    const size_t dyn = in_smem ? key_bytes : 0;
+    if (dyn > 48 * 1024 &&
+        cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn) !=
+            cudaSuccess)
+        return ECHO_ERR_CUDA;
+    {
+        LaunchScope ls(ECHO_K_TOPK, NT, K, 0, st);
+        topk_kernel<<<1, kTopkThreads, dyn, st>>>(sc, NT, K, in_smem, idx);
+    }
+    return last_launch_status();
+}

@@ -1,0 +1,282 @@
+"""ctypes binding of libechocache.so (include/echocache.h), same names as the C entry points.
+
+Argument marshalling only: every step of the cached DiT step runs in the
+library's CUDA kernels.  Tensors are torch CUDA tensors (device memory and
+streams come from PyTorch); outputs are allocated here when not given.  There
+is no fallback: a missing library or a non-sm_103 device raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libechocache.so")
+
+ECHO_OK = 0
+ECHO_BF16, ECHO_F32 = 0, 1
+MODE_ENERGY_DRIFT, MODE_SEGMENT, MODE_DRIFT_ONLY = 0, 1, 2
+
+_c = ctypes
+_vp, _i32, _i64, _sz, _f32 = _c.c_void_p, _c.c_int32, _c.c_int64, _c.c_size_t, _c.c_float
+
+
+class EchoError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        self.status = status
+        super().__init__(f"{fn} failed: {status_str(status)} ({status})")
+
+
+class SelectParams(_c.Structure):
+    _fields_ = [("lambda_", _f32), ("xi", _f32), ("mode", _i32)]
+
+
+class BlockDims(_c.Structure):
+    _fields_ = [("T", _i32), ("N", _i32), ("D", _i32), ("H", _i32), ("d", _i32), ("F", _i32),
+                ("Lc", _i32)]
+
+
+class BlockWeightsC(_c.Structure):
+    _fields_ = [(n, _vp) for n in ("Wq", "bq", "Wkv", "bkv", "Wo", "bo", "Wqc", "bqc", "Woc",
+                                   "boc", "W1", "b1", "W2", "b2", "KVc")]
+
+
+_SIGS = {
+    "echo_status_str": (_c.c_char_p, [_i32]),
+    "echo_get_device_error": (_i32, [_vp]),
+    "echo_audio_energy": (_i32, [_vp, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _vp]),
+    "echo_select_workspace_size": (_sz, [_i32, _i32]),
+    "echo_select": (_i32, [_vp, _i32, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32,
+                           _c.POINTER(SelectParams), _vp, _c.POINTER(_i32), _vp, _vp, _sz, _vp]),
+    "echo_workspace_size": (_sz, [_c.POINTER(BlockDims), _i32]),
+    "echo_precompute_cross_kv": (_i32, [_vp, _vp, _vp, _i32, _i32, _vp, _vp]),
+    "echo_block_step": (_i32, [_c.POINTER(BlockWeightsC), _c.POINTER(BlockDims), _vp, _vp, _i32,
+                               _vp, _vp, _vp, _vp, _sz, _vp]),
+    "echo_cache_quant": (_i32, [_vp, _i32, _vp, _i32, _i32, _vp, _vp, _vp]),
+    "echo_cache_dequant": (_i32, [_vp, _vp, _vp, _i32, _i32, _vp, _i32, _vp]),
+    "echo_linear": (_i32, [_vp, _i64, _i32, _i32, _vp, _vp, _i32, _i32, _vp, _i32, _vp, _vp, _i64,
+                           _i32, _vp]),
+    "echo_attention": (_i32, [_vp, _i64, _vp, _vp, _i64, _i32, _i32, _i32, _i32, _vp, _i64, _vp]),
+    "echo_layernorm": (_i32, [_vp, _i32, _vp, _i32, _i32, _vp, _vp]),
+    "echo_launch_count": (_c.c_uint64, []),
+    "echo_profile_enable": (_i32, [_i32]),
+    "echo_profile_read": (_i32, [_i32, _vp, _vp, _vp, _vp, _vp]),
+    "echo_kernel_name": (_c.c_char_p, [_i32]),
+}
+
+_LIB = None
+
+
+def lib():
+    """Load the in-tree library (built by __graft_entry__.build() or build.py)."""
+    global _LIB
+    if _LIB is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it first (python -c "
+                               "'import __graft_entry__ as g; g.build()')")
+        L = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in _SIGS.items():
+            f = getattr(L, name)
+            f.restype, f.argtypes = res, args
+        _LIB = L
+    return _LIB
+
+
+def status_str(s: int) -> str:
+    return lib().echo_status_str(int(s)).decode()
+
+
+def _check(fn: str, s: int):
+    if s != ECHO_OK:
+        raise EchoError(fn, s)
+
+
+def _p(t):
+    return None if t is None else _vp(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return _vp(s.cuda_stream)
+
+
+def _dtype(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return ECHO_BF16
+    if t.dtype == torch.float32:
+        return ECHO_F32
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _dev(t: torch.Tensor, name: str):
+    if not (t.is_cuda and t.is_contiguous()):
+        raise ValueError(f"{name} must be a contiguous CUDA tensor")
+
+
+# ---------------------------------------------------------------------------
+def echo_get_device_error(stream=None) -> int:
+    return lib().echo_get_device_error(_stream(stream))
+
+
+def echo_audio_energy(audio: torch.Tensor, T: int, n_fft: int = 512, hop: int = 160,
+                      n_bands: int = 8, band=None, seg=None, stream=None):
+    _dev(audio, "audio")
+    band = band if band is not None else torch.empty(T, n_bands, device=audio.device)
+    seg = seg if seg is not None else torch.empty(T, device=audio.device)
+    _check("echo_audio_energy", lib().echo_audio_energy(
+        _p(audio), audio.numel(), T, n_fft, hop, n_bands, _p(band), _p(seg), _stream(stream)))
+    return band, seg
+
+
+def echo_select_workspace_size(T: int, N: int) -> int:
+    return lib().echo_select_workspace_size(T, N)
+
+
+def echo_select(x, cache_q, cache_scale, seg_energy, T: int, N: int, ratio_num: int,
+                ratio_den: int, lam: float = 0.1, xi: float = 1e-6, mode: int = MODE_ENERGY_DRIFT,
+                idx=None, scores=None, workspace=None, stream=None):
+    """Returns (idx[:K] int32, K, scores or None)."""
+    for t, n in ((x, "x"), (cache_q, "cache_q"), (cache_scale, "cache_scale"),
+                 (seg_energy, "seg_energy")):
+        _dev(t, n)
+    NT, D = x.shape
+    idx = idx if idx is not None else torch.empty(NT, dtype=torch.int32, device=x.device)
+    if scores is None and workspace is None:
+        workspace = torch.empty(echo_select_workspace_size(T, N), dtype=torch.uint8, device=x.device)
+    prm = SelectParams(lam, xi, mode)
+    K = _i32(0)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check("echo_select", lib().echo_select(
+        _p(x), _dtype(x), _p(cache_q), _p(cache_scale), _p(seg_energy), T, N, D, ratio_num,
+        ratio_den, _c.byref(prm), _p(idx), _c.byref(K), _p(scores), _p(workspace), ws_bytes,
+        _stream(stream)))
+    return idx[:K.value], K.value, scores
+
+
+def echo_workspace_size(dims: BlockDims, K_max: int) -> int:
+    return lib().echo_workspace_size(_c.byref(dims), K_max)
+
+
+def echo_precompute_cross_kv(cond, Wkvc, bkvc, KVc=None, stream=None):
+    Lc, D = cond.shape
+    KVc = KVc if KVc is not None else torch.empty(Lc, 2 * D, dtype=torch.bfloat16, device=cond.device)
+    _check("echo_precompute_cross_kv", lib().echo_precompute_cross_kv(
+        _p(cond), _p(Wkvc), _p(bkvc), Lc, D, _p(KVc), _stream(stream)))
+    return KVc
+
+
+def echo_block_step(weights: "DeviceBlock", dims: BlockDims, x, idx, K: int, cache_q, cache_scale,
+                    y=None, workspace=None, stream=None):
+    y = y if y is not None else torch.empty_like(x)
+    if workspace is None:
+        workspace = torch.empty(echo_workspace_size(dims, K), dtype=torch.uint8, device=x.device)
+    _check("echo_block_step", lib().echo_block_step(
+        _c.byref(weights.cstruct), _c.byref(dims), _p(x), _p(idx) if K > 0 else None, K,
+        _p(cache_q), _p(cache_scale), _p(y), _p(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
+    return y
+
+
+def echo_cache_quant(src, rows, q, scale, stream=None):
+    n, D = src.shape
+    _check("echo_cache_quant", lib().echo_cache_quant(
+        _p(src), _dtype(src), _p(rows), n, D, _p(q), _p(scale), _stream(stream)))
+
+
+def echo_cache_dequant(q, scale, rows=None, dtype=torch.bfloat16, out=None, stream=None):
+    n = q.shape[0] if rows is None else rows.numel()
+    D = q.shape[1]
+    out = out if out is not None else torch.empty(n, D, dtype=dtype, device=q.device)
+    _check("echo_cache_dequant", lib().echo_cache_dequant(
+        _p(q), _p(scale), _p(rows), n, D, _p(out), _dtype(out), _stream(stream)))
+    return out
+
+
+def echo_linear(A, W, bias=None, act: int = 0, resid=None, resid_rows=None,
+                out_dtype=torch.bfloat16, out=None, stream=None):
+    M, Kd = A.shape
+    N = W.shape[0]
+    out = out if out is not None else torch.empty(M, N, dtype=out_dtype, device=A.device)
+    rt = _dtype(resid) if resid is not None else ECHO_BF16
+    _check("echo_linear", lib().echo_linear(
+        _p(A), A.stride(0), M, Kd, _p(W), _p(bias), N, act, _p(resid), rt, _p(resid_rows),
+        _p(out), out.stride(0), _dtype(out), _stream(stream)))
+    return out
+
+
+def echo_attention(Q, K, V, H: int, d: int, out=None, stream=None):
+    """Q [M, >=H d] (row stride Q.stride(0)), K and V [L, *] sharing one row stride."""
+    M, L = Q.shape[0], K.shape[0]
+    if K.stride(0) != V.stride(0):
+        raise ValueError("K and V must share a row stride")
+    out = out if out is not None else torch.empty(M, H * d, dtype=torch.bfloat16, device=Q.device)
+    _check("echo_attention", lib().echo_attention(
+        _p(Q), Q.stride(0), _p(K), _p(V), K.stride(0), M, L, H, d, _p(out), out.stride(0),
+        _stream(stream)))
+    return out
+
+
+def echo_layernorm(inp, rows=None, out=None, stream=None):
+    n = inp.shape[0] if rows is None else rows.numel()
+    D = inp.shape[1]
+    out = out if out is not None else torch.empty(n, D, dtype=torch.bfloat16, device=inp.device)
+    _check("echo_layernorm", lib().echo_layernorm(
+        _p(inp), _dtype(inp), _p(rows), n, D, _p(out), _stream(stream)))
+    return out
+
+
+def echo_launch_count() -> int:
+    return int(lib().echo_launch_count())
+
+
+def echo_profile_enable(on: bool = True):
+    _check("echo_profile_enable", lib().echo_profile_enable(1 if on else 0))
+
+
+def echo_kernel_name(kind: int) -> str:
+    return lib().echo_kernel_name(int(kind)).decode()
+
+
+def echo_profile_read(max_records: int = 65536):
+    """List of (kernel name, m, n, k, ms) for every launch recorded since the last read."""
+    import numpy as np
+    kinds = np.zeros(max_records, np.int32)
+    m, n, k = (np.zeros(max_records, np.int64) for _ in range(3))
+    ms = np.zeros(max_records, np.float32)
+    cnt = lib().echo_profile_read(max_records, kinds.ctypes.data, m.ctypes.data, n.ctypes.data,
+                                  k.ctypes.data, ms.ctypes.data)
+    if cnt < 0:
+        raise EchoError("echo_profile_read", 4)
+    return [(echo_kernel_name(kinds[i]), int(m[i]), int(n[i]), int(k[i]), float(ms[i]))
+            for i in range(cnt)]
+
+
+# ---------------------------------------------------------------------------
+@dataclass
+class DeviceBlock:
+    """One block's parameters resident on the device, in the layout the C ABI takes."""
+    tensors: dict
+    cstruct: BlockWeightsC
+
+    @staticmethod
+    def from_host(W: dict, cond, device="cuda", stream=None) -> "DeviceBlock":
+        """W: nn.Linear-convention arrays (numpy or torch, bf16 values); cond [Lc, D]."""
+        bf = lambda a: torch.as_tensor(a).to(device=device, dtype=torch.bfloat16).contiguous()
+        t = {
+            "Wq": bf(W["Wq"]), "bq": bf(W["bq"]),
+            "Wkv": torch.cat([bf(W["Wk"]), bf(W["Wv"])]).contiguous(),
+            "bkv": torch.cat([bf(W["bk"]), bf(W["bv"])]).contiguous(),
+            "Wo": bf(W["Wo"]), "bo": bf(W["bo"]),
+            "Wqc": bf(W["Wqc"]), "bqc": bf(W["bqc"]),
+            "Woc": bf(W["Woc"]), "boc": bf(W["boc"]),
+            "W1": bf(W["W1"]), "b1": bf(W["b1"]),
+            "W2": bf(W["W2"]), "b2": bf(W["b2"]),
+        }
+        Wkvc = torch.cat([bf(W["Wkc"]), bf(W["Wvc"])]).contiguous()
+        bkvc = torch.cat([bf(W["bkc"]), bf(W["bvc"])]).contiguous()
+        t["KVc"] = echo_precompute_cross_kv(bf(cond), Wkvc, bkvc, stream=stream)
+        c = BlockWeightsC(*[_p(t[n]) for n, _ in BlockWeightsC._fields_])
+        return DeviceBlock(t, c)
