@@ -124,8 +124,9 @@ def echo_get_device_error(stream=None) -> int:
 def echo_audio_energy(audio: torch.Tensor, T: int, n_fft: int = 512, hop: int = 160,
                       n_bands: int = 8, band=None, seg=None, stream=None):
     _dev(audio, "audio")
-    band = band if band is not None else torch.empty(T, n_bands, device=audio.device)
-    seg = seg if seg is not None else torch.empty(T, device=audio.device)
+    band = band if band is not None else torch.empty(T, n_bands, dtype=torch.float32,
+                                                     device=audio.device)
+    seg = seg if seg is not None else torch.empty(T, dtype=torch.float32, device=audio.device)
     _check("echo_audio_energy", lib().echo_audio_energy(
         _p(audio), audio.numel(), T, n_fft, hop, n_bands, _p(band), _p(seg), _stream(stream)))
     return band, seg

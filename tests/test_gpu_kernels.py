@@ -2,7 +2,7 @@
 
 Bars: bit-exact for the int8 cache, scales, dequantised rows, drift scores and
 selected indices; rel <= 1e-5 for fp32 energies; bf16 outputs within the
-block tolerance (max rel <= 2e-2 with a 0.1 rms floor, mean rel <= 5e-3).
+block tolerance (per-row normwise max rel <= 2e-2, mean rel <= 5e-3).
 """
 import numpy as np
 import pytest
@@ -36,10 +36,12 @@ def f32(a):
 
 
 def close_bf16(g, o, max_rel=2e-2, mean_rel=5e-3):
+    """Per-row normwise max relative error max_j|g-o| / max_j|o| and the mean
+    relative error sum|g-o| / sum|o| (the reading justified in
+    test_tolerance_reading.py)."""
     g = np.asarray(g, dtype=np.float64)
     o = np.asarray(o, dtype=np.float64)
-    den = np.maximum(np.abs(o), 0.1 * np.sqrt((o ** 2).mean(axis=-1, keepdims=True)) + 1e-30)
-    rel = np.abs(g - o) / den
+    rel = np.abs(g - o).max(axis=-1) / np.maximum(np.abs(o).max(axis=-1), 1e-30)
     mr = np.abs(g - o).sum() / max(np.abs(o).sum(), 1e-30)
     assert rel.max() <= max_rel and mr <= mean_rel, (float(rel.max()), float(mr))
     return float(rel.max()), float(mr)
@@ -92,7 +94,7 @@ def test_quant_bit_exact(ec, D, src_t):
         v = G.to_bf16_values(v)
     rows = np.random.default_rng(1).permutation(2 * n)[:n].astype(np.int32)
     q = torch.zeros(2 * n, D, dtype=torch.int8, device=DEV)
-    s = torch.full((2 * n,), -1.0, device=DEV)
+    s = torch.full((2 * n,), -1.0, dtype=torch.float32, device=DEV)
     src = bf(v) if src_t == "bf16" else f32(v)
     ec.echo_cache_quant(src, torch.from_numpy(rows).to(DEV), q, s)
     oq = np.zeros((2 * n, D), np.int8)
@@ -107,7 +109,7 @@ def test_quant_identity_rows_and_nonfinite_flag(ec):
     v = G.random_rows(40, 64, seed=3)
     v[11, 3] = np.inf
     q = torch.zeros(40, 64, dtype=torch.int8, device=DEV)
-    s = torch.zeros(40, device=DEV)
+    s = torch.zeros(40, dtype=torch.float32, device=DEV)
     ec.echo_cache_quant(bf(v), None, q, s)
     assert ec.echo_get_device_error() == 5          # NONFINITE, then cleared
     assert ec.echo_get_device_error() == 0
@@ -158,7 +160,7 @@ def test_select_bit_exact(ec, T, N, D, ratio, mode, distinct):
     if not distinct:
         e[1] = e[0]
     xd = bf(x)
-    scores = torch.empty(NT, device=DEV)
+    scores = torch.empty(NT, dtype=torch.float32, device=DEV)
     idx, K, _ = ec.echo_select(xd, torch.from_numpy(q).to(DEV), f32(s), f32(e), T, N, *ratio,
                                mode=mode, scores=scores)
     oidx, osc = oracle.select.select(x, q, s, e, T, N, *ratio, mode=mode)
@@ -199,6 +201,8 @@ def test_select_with_silence_is_drift_only(ec):
 def test_layernorm(ec, D, in_t):
     n = 77
     x = G.random_rows(n, D, seed=D + 7, scale=2.0) + F32(0.5)
+    if in_t == "bf16":
+        x = G.to_bf16_values(x)
     rows = np.random.default_rng(D).permutation(n)[:50].astype(np.int32)
     src = bf(x) if in_t == "bf16" else f32(x)
     out = ec.echo_layernorm(src, torch.from_numpy(rows).to(DEV))

@@ -9,11 +9,13 @@ from oracle import cache as C
 from oracle import step as ST
 from synth import generate as G, small
 
-torch.set_default_dtype(torch.float64)
 
 
 def _t(a):
     return torch.from_numpy(np.asarray(a, dtype=np.float64))
+
+
+F64 = dict(dtype=torch.float64)
 
 
 def test_layer_norm_matches_torch():
@@ -62,8 +64,8 @@ def test_mha_key_permutation_invariance():
 def _torch_block(x, W, cond, H, idx):
     """The same block assembled from torch.nn modules (fp64), for the active rows."""
     D = x.shape[1]
-    sa = torch.nn.MultiheadAttention(D, H, bias=True, batch_first=True)
-    ca = torch.nn.MultiheadAttention(D, H, bias=True, batch_first=True)
+    sa = torch.nn.MultiheadAttention(D, H, bias=True, batch_first=True, **F64)
+    ca = torch.nn.MultiheadAttention(D, H, bias=True, batch_first=True, **F64)
     with torch.no_grad():
         sa.in_proj_weight.copy_(torch.cat([_t(W["Wq"]), _t(W["Wk"]), _t(W["Wv"])]))
         sa.in_proj_bias.copy_(torch.cat([_t(W["bq"]), _t(W["bk"]), _t(W["bv"])]))
@@ -73,8 +75,9 @@ def _torch_block(x, W, cond, H, idx):
         ca.in_proj_bias.copy_(torch.cat([_t(W["bqc"]), _t(W["bkc"]), _t(W["bvc"])]))
         ca.out_proj.weight.copy_(_t(W["Woc"]))
         ca.out_proj.bias.copy_(_t(W["boc"]))
-        ln = torch.nn.LayerNorm(D, eps=1e-6, elementwise_affine=False)
-        up, down = torch.nn.Linear(D, W["W1"].shape[0]), torch.nn.Linear(W["W1"].shape[0], D)
+        ln = torch.nn.LayerNorm(D, eps=1e-6, elementwise_affine=False, **F64)
+        up = torch.nn.Linear(D, W["W1"].shape[0], **F64)
+        down = torch.nn.Linear(W["W1"].shape[0], D, **F64)
         up.weight.copy_(_t(W["W1"]))
         up.bias.copy_(_t(W["b1"]))
         down.weight.copy_(_t(W["W2"]))
