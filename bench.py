@@ -193,13 +193,13 @@ def oracle_sample(w, audio, W, cond, x1, q, s, rnum, rden, budget_s=25.0):
     idx, _ = oracle.select.select(x1, q, s, e32, w.T, w.N, rnum, rden)
     t["select"] = time.perf_counter() - t0
     K = len(idx)
-    s_kv = min(w.NT, 1024)
+    s_kv = min(w.NT, 4096)
     t0 = time.perf_counter()
     oracle.block.self_kv(x1[:s_kv], W)
     t["kv_sample"] = time.perf_counter() - t0
     Kc, Vc = oracle.block.cross_kv(cond, W)
     kv_stand_in = x1.astype(np.float64)      # any [NT, D] array: only the timing is used
-    s_a = min(K, 32)
+    s_a = min(K, 128)
     t0 = time.perf_counter()
     oracle.block.active_rows(x1, idx[:s_a], W, w.H, kv_stand_in, kv_stand_in, Kc, Vc)
     t["active_sample"] = time.perf_counter() - t0
