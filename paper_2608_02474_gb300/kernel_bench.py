@@ -1,0 +1,117 @@
+"""Run one kernel of the library at one shape, for timing and ncu captures.
+
+    python -m paper_2608_02474_gb300.kernel_bench --kernel gemm --M 32760 --N 10240 --K 5120
+    python -m paper_2608_02474_gb300.kernel_bench --kernel attention --M 6552 --L 32760 --H 40 --d 128
+    python -m paper_2608_02474_gb300.kernel_bench --kernel drift --T 21 --N 1560 --D 5120
+    python -m paper_2608_02474_gb300.kernel_bench --kernel merge --T 21 --N 1560 --D 5120 --K 6552
+
+Inputs are seeded random device tensors of the right shapes (values do not
+change the work of these kernels).  Prints the mean time per launch over
+--iters launches after --warmup launches, measured with CUDA events on the
+launching stream, plus the achieved TFLOP/s or GB/s.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+
+import torch
+
+from . import echocache as ec
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--kernel", required=True,
+                    choices=["gemm", "attention", "drift", "select", "merge", "quant", "layernorm"])
+    ap.add_argument("--M", type=int, default=6552)
+    ap.add_argument("--N", type=int, default=5120)
+    ap.add_argument("--K", type=int, default=5120)
+    ap.add_argument("--L", type=int, default=32760)
+    ap.add_argument("--H", type=int, default=40)
+    ap.add_argument("--d", type=int, default=128)
+    ap.add_argument("--T", type=int, default=21)
+    ap.add_argument("--D", type=int, default=5120)
+    ap.add_argument("--act", type=int, default=0)
+    ap.add_argument("--iters", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=1)
+    a = ap.parse_args()
+
+    dev = torch.device("cuda")
+    g = torch.Generator(device=dev).manual_seed(0)
+    rn = lambda *s: torch.randn(*s, generator=g, device=dev, dtype=torch.float32)
+
+    if a.kernel == "gemm":
+        A = rn(a.M, a.K).to(torch.bfloat16)
+        W = (rn(a.N, a.K) * 0.02).to(torch.bfloat16)
+        b = (rn(a.N) * 0.02).to(torch.bfloat16)
+        out = torch.empty(a.M, a.N, dtype=torch.bfloat16, device=dev)
+        run = lambda: ec.echo_linear(A, W, b, act=a.act, out=out)
+        work, unit = 2.0 * a.M * a.N * a.K, "TFLOP/s"
+    elif a.kernel == "attention":
+        D = a.H * a.d
+        Q = rn(a.M, D).to(torch.bfloat16)
+        KV = rn(a.L, 2 * D).to(torch.bfloat16)
+        out = torch.empty(a.M, D, dtype=torch.bfloat16, device=dev)
+        run = lambda: ec.echo_attention(Q, KV[:, :D], KV[:, D:], a.H, a.d, out=out)
+        work, unit = 4.0 * a.M * a.L * D, "TFLOP/s"
+    elif a.kernel in ("drift", "select"):
+        NT = a.T * a.N
+        x = rn(NT, a.D).to(torch.bfloat16)
+        q = torch.randint(-127, 128, (NT, a.D), generator=g, device=dev, dtype=torch.int8)
+        s = torch.rand(NT, generator=g, device=dev) * 0.05
+        e = torch.rand(a.T, generator=g, device=dev)
+        idx = torch.empty(NT, dtype=torch.int32, device=dev)
+        sc = torch.empty(NT, dtype=torch.float32, device=dev)
+        run = lambda: ec.echo_select(x, q, s, e, a.T, a.N, 1, 5, idx=idx, scores=sc)
+        work, unit = NT * (3.0 * a.D + 8), "GB/s"
+    elif a.kernel in ("merge", "quant"):
+        NT = a.T * a.N
+        D = a.D
+        q = torch.randint(-127, 128, (NT, D), generator=g, device=dev, dtype=torch.int8)
+        s = torch.rand(NT, generator=g, device=dev) * 0.05
+        perm = torch.randperm(NT, generator=g, device=dev)[:a.K]
+        idx = torch.sort(perm).values.to(torch.int32)
+        yact = rn(a.K, D).to(torch.bfloat16)
+        if a.kernel == "quant":
+            run = lambda: ec.echo_cache_quant(yact, idx, q, s)
+            work = a.K * (3.0 * D + 8)
+        else:
+            # K = 0 block step is exactly the merge kernel plus the row map
+            dims = ec.BlockDims(a.T, a.N, D, a.H, a.d, 4096, 16)
+            y = torch.empty(NT, D, dtype=torch.bfloat16, device=dev)
+            fake = torch.zeros(64, dtype=torch.bfloat16, device=dev)
+
+            class _W:
+                cstruct = ec.BlockWeightsC(*([fake.data_ptr()] * 15))
+            ws = torch.empty(ec.echo_workspace_size(dims, 0), dtype=torch.uint8, device=dev)
+            x = torch.empty(NT, D, dtype=torch.bfloat16, device=dev)
+            run = lambda: ec.echo_block_step(_W, dims, x, None, 0, q, s, y=y, workspace=ws)
+            work = NT * (D + 4.0) + NT * 2.0 * D + 4.0 * NT
+        unit = "GB/s"
+    else:  # layernorm
+        NT = a.T * a.N
+        x = rn(NT, a.D).to(torch.bfloat16)
+        out = torch.empty_like(x)
+        run = lambda: ec.echo_layernorm(x, out=out)
+        work, unit = NT * 4.0 * a.D, "GB/s"
+
+    for _ in range(a.warmup):
+        run()
+    torch.cuda.synchronize()
+    st = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    for _ in range(a.iters):
+        run()
+    e1.record(st)
+    torch.cuda.synchronize()
+    assert ec.echo_get_device_error() == 0
+    ms = e0.elapsed_time(e1) / a.iters
+    rate = work / (ms * 1e-3) / (1e12 if unit == "TFLOP/s" else 1e9)
+    print(json.dumps({"kernel": a.kernel, "ms": round(ms, 4), unit: round(rate, 1),
+                      "args": vars(a)}))
+
+
+if __name__ == "__main__":
+    main()
