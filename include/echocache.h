@@ -157,6 +157,33 @@ echo_status echo_select(const void *x, echo_dtype xt, const int8_t *cache_q,
                         int32_t *idx, int32_t *K_out, float *scores,
                         void *workspace, size_t ws_bytes, echo_stream_t stream);
 
+/* No counterpart in the paper: a variant of echo_select for callers that
+ * cannot allocate device memory.  Some callers own no allocator at all: code
+ * running inside a host application that reserves all device memory up front
+ * and forbids cudaMalloc after start-up, or code on a latency-critical thread
+ * where cudaMalloc/cudaFree would synchronise the whole device.  This entry
+ * point takes no workspace and allocates nothing: the drift scores live in a
+ * library-owned static device array of ECHO_SELECT_STATIC_MAX_TOKENS floats
+ * (256 KiB), which every GPU that loads the library holds until the process
+ * exits.
+ *   Arguments and results are those of echo_select, without scores and
+ *   workspace; T * N must not exceed ECHO_SELECT_STATIC_MAX_TOKENS, otherwise
+ *   ECHO_ERR_WORKSPACE is returned and nothing is enqueued.
+ *   The first call on a device looks up that device's address of the array
+ *   (once, with the device current); make that first call before any CUDA
+ *   stream capture.
+ *   All calls on a device share the one array and it keeps the last call's
+ *   scores; nothing in it needs to start at zero, because every score the
+ *   top-K reads is written first by the same call.  Calls whose work overlaps
+ *   on the GPU (different streams, or different host threads without
+ *   ordering) race on the array: order them on one stream. */
+#define ECHO_SELECT_STATIC_MAX_TOKENS 65536
+echo_status echo_select_static(const void *x, echo_dtype xt, const int8_t *cache_q,
+                               const float *cache_scale, const float *seg_energy,
+                               int32_t T, int32_t N, int32_t D, int32_t ratio_num,
+                               int32_t ratio_den, const echo_select_params *p,
+                               int32_t *idx, int32_t *K_out, echo_stream_t stream);
+
 /* Bytes of workspace echo_block_step needs for dims and up to K_max active
  * tokens (also enough for echo_precompute_cross_kv). */
 size_t echo_workspace_size(const echo_block_dims *dims, int32_t K_max);

@@ -9,6 +9,8 @@
 // topk_kernel: one CTA radix-selects the K-th largest 32-bit key (11/11/10-bit
 //   digits), then compacts in index order, taking keys equal to the threshold
 //   from the lowest index up.
+#include <mutex>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -324,6 +326,95 @@ extern "C" echo_status echo_select(const void *x, echo_dtype xt, const int8_t *c
     const size_t key_bytes = (size_t)NT * sizeof(uint32_t);
     const size_t max_dyn = 200 * 1024;
     const int in_smem = key_bytes <= max_dyn ? 1 : 0;
+    const size_t dyn = in_smem ? key_bytes : 0;
+    if (dyn > 48 * 1024 &&
+        cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn) !=
+            cudaSuccess)
+        return ECHO_ERR_CUDA;
+    {
+        LaunchScope ls(ECHO_K_TOPK, NT, K, 0, st);
+        topk_kernel<<<1, kTopkThreads, dyn, st>>>(sc, NT, K, in_smem, idx);
+    }
+    return last_launch_status();
+}
+
+// ---------------------------------------------------------------------------
+// echo_select_static: the same selection for callers that cannot allocate.
+// The scores live in this file-scope device array instead of a workspace.
+// Host code must not pass `g_select_scratch` itself to a kernel (on the host
+// it is only a stand-in symbol); the device address is looked up once per
+// device with cudaGetSymbolAddress and cached.
+// ---------------------------------------------------------------------------
+static __device__ __align__(256) float g_select_scratch[ECHO_SELECT_STATIC_MAX_TOKENS];
+
+namespace {
+
+constexpr int kScratchDevices = 64;
+float *g_scratch_ptr[kScratchDevices] = {};
+std::mutex g_scratch_mu;
+
+// Address of this device's scratch array (the current device), or nullptr.
+float *select_scratch_for_current_device() {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kScratchDevices) return nullptr;
+    std::lock_guard<std::mutex> lk(g_scratch_mu);
+    if (!g_scratch_ptr[dev]) {
+        float *ptr = nullptr;
+        if (cudaGetSymbolAddress(reinterpret_cast<void **>(&ptr), g_select_scratch) != cudaSuccess ||
+            !ptr)
+            return nullptr;
+        g_scratch_ptr[dev] = ptr;
+    }
+    return g_scratch_ptr[dev];
+}
+
+}  // namespace
+
+extern "C" echo_status echo_select_static(const void *x, echo_dtype xt, const int8_t *cache_q,
+                                          const float *cache_scale, const float *seg_energy,
+                                          int32_t T, int32_t N, int32_t D, int32_t ratio_num,
+                                          int32_t ratio_den, const echo_select_params *p,
+                                          int32_t *idx, int32_t *K_out, echo_stream_t stream) {
+    using namespace echo;
+    if (!x || !cache_q || !cache_scale || !seg_energy || !idx || !K_out) return ECHO_ERR_INVALID_ARG;
+    if (xt != ECHO_BF16 && xt != ECHO_F32) return ECHO_ERR_INVALID_ARG;
+    if (!aligned16(x) || !aligned16(cache_q) || !aligned16(cache_scale) || !aligned16(seg_energy) ||
+        !aligned16(idx))
+        return ECHO_ERR_INVALID_ARG;
+    echo_select_params prm = {0.1f, 1e-6f, ECHO_MODE_ENERGY_DRIFT};
+    if (p) prm = *p;
+    if (prm.mode < 0 || prm.mode > 2 || !(prm.xi > 0.f) || !(prm.lambda >= 0.f) ||
+        !(prm.lambda <= 1.f))
+        return ECHO_ERR_INVALID_ARG;
+    if (T < 1 || N < 1 || D < 8 || D % 8 || ratio_den < 1 || ratio_num < 0 || ratio_num > ratio_den)
+        return ECHO_ERR_SHAPE;
+    const int64_t NT64 = (int64_t)T * N;
+    if (NT64 > ECHO_SELECT_STATIC_MAX_TOKENS) return ECHO_ERR_WORKSPACE;
+    const int NT = (int)NT64;
+    const int K = (int)(((int64_t)ratio_num * NT + ratio_den - 1) / ratio_den);
+    if (!device_supported()) return ECHO_ERR_UNSUPPORTED;
+    float *sc = select_scratch_for_current_device();
+    if (!sc) return ECHO_ERR_CUDA;
+    *K_out = K;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    int *err = device_error_ptr();
+
+    const int warps = kDriftThreads / 32;
+    const int grid = (NT + warps - 1) / warps;
+    {
+        LaunchScope ls(ECHO_K_DRIFT, NT, D, 0, st);
+        if (xt == ECHO_BF16)
+            drift_kernel<__nv_bfloat16><<<grid, kDriftThreads, 0, st>>>(
+                static_cast<const __nv_bfloat16 *>(x), cache_q, cache_scale, seg_energy, T, N, NT,
+                D, prm.lambda, prm.xi, prm.mode, sc, err);
+        else
+            drift_kernel<float><<<grid, kDriftThreads, 0, st>>>(
+                static_cast<const float *>(x), cache_q, cache_scale, seg_energy, T, N, NT, D,
+                prm.lambda, prm.xi, prm.mode, sc, err);
+    }
+    if (last_launch_status() != ECHO_OK) return ECHO_ERR_CUDA;
+    const size_t key_bytes = (size_t)NT * sizeof(uint32_t);
+    const int in_smem = key_bytes <= 200 * 1024 ? 1 : 0;
     const size_t dyn = in_smem ? key_bytes : 0;
     if (dyn > 48 * 1024 &&
         cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn) !=

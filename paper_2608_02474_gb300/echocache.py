@@ -51,6 +51,8 @@ _SIGS = {
     "echo_select_workspace_size": (_sz, [_i32, _i32]),
     "echo_select": (_i32, [_vp, _i32, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32,
                            _c.POINTER(SelectParams), _vp, _c.POINTER(_i32), _vp, _vp, _sz, _vp]),
+    "echo_select_static": (_i32, [_vp, _i32, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32,
+                                  _c.POINTER(SelectParams), _vp, _c.POINTER(_i32), _vp]),
     "echo_workspace_size": (_sz, [_c.POINTER(BlockDims), _i32]),
     "echo_precompute_cross_kv": (_i32, [_vp, _vp, _vp, _i32, _i32, _vp, _vp]),
     "echo_block_step": (_i32, [_c.POINTER(BlockWeightsC), _c.POINTER(BlockDims), _vp, _vp, _i32,
