@@ -137,18 +137,19 @@ def roofline(records, K, peaks):
     shape = max(shapes, key=lambda s: s[0] * s[1])
     avg_ms, cnt, (name, m, n, k) = shape
     flops, byts = algorithmic_work(name, m, n, k, K)
+    traffic = measured_traffic(name, [m, n, k])
     if flops is not None:
         achieved = flops / (avg_ms * 1e-3) / 1e12
         peak = peaks["bf16_tflops_sustained"]
         out = {"bound": "tensor", "kernel": name, "shape": [m, n, k], "achieved": round(achieved, 2),
                "peak": peak, "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
-               "traffic": None, "algorithmic_flops": flops, "launch_ms": round(avg_ms, 4),
+               "traffic": traffic, "algorithmic_flops": flops, "launch_ms": round(avg_ms, 4),
                "peak_source": "measured bf16_tflops_sustained"}
     else:
         achieved = byts / (avg_ms * 1e-3) / 1e9
         peak = peaks["hbm_gbs"]
         out = {"bound": "hbm", "kernel": name, "shape": [m, n, k], "achieved": round(achieved, 1),
-               "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": None,
+               "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": traffic,
                "algorithmic_bytes": byts, "launch_ms": round(avg_ms, 4),
                "peak_source": "measured hbm_gbs"}
     table = {}
@@ -161,6 +162,24 @@ def roofline(records, K, peaks):
             row["gbs"] = round(b / (ms / c * 1e-3) / 1e9, 1)
         table[f"{nm}[{m}x{n}x{k}]"] = row
     return out, table
+
+
+def measured_traffic(kernel, shape):
+    """DRAM bytes per launch from profiles/traffic.json, only while the kernel's
+    source file is unchanged since the capture (else None)."""
+    import hashlib
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    e = json.load(open(p)).get(kernel)
+    if not e or list(e["shape"]) != list(shape):
+        return None
+    src = os.path.join(ROOT, e["source"])
+    if not os.path.exists(src):
+        return None
+    if hashlib.sha256(open(src, "rb").read()).hexdigest()[:16] != e["sha256_16"]:
+        return None
+    return e["bytes"]
 
 
 def load_peaks():
