@@ -2,241 +2,322 @@
 // latents, keys and values over the complete latent set (self-attention) or the
 // audio condition tokens (cross-attention).
 //
-// Flash-style forward: one CTA per (128-query tile, head), 8 warps of 16 query
-// rows; K/V blocks of 64 keys double-buffered in swizzled shared memory by
-// cp.async; S = Q K^T and O += P V on bf16 mma.sync with fp32 accumulators;
-// online softmax in registers (exp2 with the 1/sqrt(d) scale folded in); P is
-// rounded to bf16 for the second product.  Keys beyond L are masked, queries
-// beyond M are computed on zeros and not stored.
+// Flash-style forward on the 5th-generation tensor cores.  One CTA per
+// (128-query tile, head), 8 warps:
+//   warp 0      TMA producer: the Q tile once, then 128-key blocks of K and V
+//               (128-byte swizzle, 64-column boxes) into two-stage rings;
+//   warp 1      one thread issues S_j = Q K_j^T (M 128, N 128, K d) into one of
+//               two TMEM S buffers, and O += P_j V_j (M 128, N d, K 128; V is
+//               read MN-major straight from its row-major tile) into a TMEM O
+//               accumulator, one block behind;
+//   warp 2      allocates / frees 512 TMEM columns (S0, S1, O);
+//   warps 4..7  softmax, one query row per thread (its TMEM lane): tcgen05.ld of
+//               the S row, online max, P = 2^(s*scale - m) rounded to bf16 into a
+//               swizzled shared-memory tile (the A operand of P V), row sum of the
+//               rounded P; O is rescaled in TMEM only when the running max grows
+//               by more than 2^8 (otherwise the stale max is kept, which is exact
+//               after the final division by the row sum); final O / l to bf16.
+// Keys beyond L are masked to P = 0; queries beyond M run on zero rows and are
+// not stored.  Every mbarrier wait is bounded (ECHO_ERR_TIMEOUT).
 #include "common.cuh"
 #include "internal.h"
 
 namespace {
 
-constexpr int BR = 128;       // queries per CTA
-constexpr int BC = 64;        // keys per block
-constexpr int THREADS = 256;  // 8 warps x 16 query rows
-
-ECHO_DEV void cp_async16(void *dst, const void *src, bool valid) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src),
-                 "r"(valid ? 16 : 0)
-                 : "memory");
-}
-ECHO_DEV void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-ECHO_DEV void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
-
-ECHO_DEV void ldsm_x4(uint32_t *r, const void *p) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-                 : "r"(smem_u32(p)));
-}
-ECHO_DEV void ldsm_x4_t(uint32_t *r, const void *p) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-                 : "r"(smem_u32(p)));
-}
-ECHO_DEV void mma_bf16(float *c, const uint32_t *a, uint32_t b0, uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
-        "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
-        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-
-// byte offset of (row, 16-byte chunk) in a tile with rows of DH bf16, chunk
-// index xor-swizzled by the row's low 3 bits
-template <int DH>
-ECHO_DEV uint32_t sw(int row, int chunk) {
-    return (uint32_t)(row * (DH * 2) + ((chunk ^ (row & 7)) << 4));
-}
+constexpr int BM = 128;        // queries per CTA
+constexpr int BN = 128;        // keys per block
+constexpr int KST = 2;         // K ring stages
+constexpr int VST = 2;         // V ring stages
+constexpr int THREADS = 256;
+constexpr uint32_t TMEM_COLS = 512;
+constexpr uint32_t O_COL = 256;
+constexpr int ATOM_BYTES = 128 * 128;   // one [128 rows x 64 bf16] 128B-swizzled box
+constexpr float RESCALE_LOG2 = 8.f;
 
 template <int DH>
-ECHO_DEV void load_rows(uint8_t *tile, const __nv_bfloat16 *base, int64_t ld, int row0, int nrows,
-                        int limit) {
-    constexpr int CPR = DH / 8;  // 16-byte chunks per row
-    for (int i = threadIdx.x; i < nrows * CPR; i += THREADS) {
-        const int r = i / CPR, c = i % CPR;
-        const int g = row0 + r;
-        const bool ok = g < limit;
-        const __nv_bfloat16 *src = base + (int64_t)(ok ? g : 0) * ld + c * 8;
-        cp_async16(tile + sw<DH>(r, c), src, ok);
-    }
-}
+struct Cfg {
+    static constexpr int ATOMS = DH / 64;
+    static constexpr int Q_BYTES = BM * DH * 2;
+    static constexpr int K_BYTES = BN * DH * 2;
+    static constexpr int V_BYTES = BN * DH * 2;
+    static constexpr int P_BYTES = BM * BN * 2;
+    static constexpr int SMEM = Q_BYTES + KST * K_BYTES + VST * V_BYTES + P_BYTES + 1024;
+    static constexpr uint32_t IDESC_S = idesc_bf16_f32(BM, BN);
+    static constexpr uint32_t IDESC_PV = idesc_bf16_f32(BM, DH) | (1u << 16);  // B MN-major
+};
+
+struct AttnParams {
+    int M, L;
+    float scale_log2;
+    __nv_bfloat16 *O;
+    int64_t ldo;
+    int *err;
+};
 
 template <int DH>
-__global__ void __launch_bounds__(THREADS)
-attn_kernel(const __nv_bfloat16 *__restrict__ Q, int64_t ldq, const __nv_bfloat16 *__restrict__ K,
-            const __nv_bfloat16 *__restrict__ V, int64_t ldkv, int M, int L,
-            __nv_bfloat16 *__restrict__ O, int64_t ldo, float scale_log2) {
-    extern __shared__ __align__(128) uint8_t sm[];
-    uint8_t *Qs = sm;
-    uint8_t *Ks = Qs + BR * DH * 2;           // [2][BC][DH]
-    uint8_t *Vs = Ks + 2 * BC * DH * 2;       // [2][BC][DH]
-    constexpr int KV_TILE = BC * DH * 2;
+__global__ void __launch_bounds__(THREADS, 1)
+attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+               const __grid_constant__ CUtensorMap tmV, const AttnParams p) {
+    using C = Cfg<DH>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                ~static_cast<uintptr_t>(1023));
+    uint8_t *Qs = smem;
+    uint8_t *Ks = Qs + C::Q_BYTES;
+    uint8_t *Vs = Ks + KST * C::K_BYTES;
+    uint8_t *Ps = Vs + VST * C::V_BYTES;
 
-    const int h = blockIdx.y;
-    const int q0 = blockIdx.x * BR;
+    __shared__ __align__(8) uint64_t q_full, k_full[KST], k_empty[KST], v_full[VST], v_empty[VST];
+    __shared__ __align__(8) uint64_t s_full[2], s_free[2], p_full, pv_done, drain;
+    __shared__ uint32_t tmem_slot;
+    __shared__ int abort_flag;
+
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const __nv_bfloat16 *Qh = Q + h * DH;
-    const __nv_bfloat16 *Kh = K + h * DH;
-    const __nv_bfloat16 *Vh = V + h * DH;
-    const int nkb = (L + BC - 1) / BC;
+    const int h = blockIdx.y;
+    const int q0 = blockIdx.x * BM;
+    const int nb = (p.L + BN - 1) / BN;
 
-    load_rows<DH>(Qs, Qh, ldq, q0, BR, M);
-    load_rows<DH>(Ks, Kh, ldkv, 0, BC, L);
-    load_rows<DH>(Vs, Vh, ldkv, 0, BC, L);
-    cp_async_commit();
-    cp_async_wait_all();
-    __syncthreads();
-
-    // Q fragments of this warp's 16 rows, all DH columns
-    uint32_t qf[DH / 16][4];
-    {
-        const int r = warp * 16 + (lane & 7) + 8 * ((lane >> 3) & 1);
-#pragma unroll
-        for (int ks = 0; ks < DH / 16; ++ks) {
-            const int c = ks * 2 + (lane >> 4);
-            ldsm_x4(qf[ks], Qs + sw<DH>(r, c));
-        }
+    if (threadIdx.x == 0) {
+        mbar_init(&q_full, 1);
+        for (int i = 0; i < KST; ++i) { mbar_init(&k_full[i], 1); mbar_init(&k_empty[i], 1); }
+        for (int i = 0; i < VST; ++i) { mbar_init(&v_full[i], 1); mbar_init(&v_empty[i], 1); }
+        for (int i = 0; i < 2; ++i) { mbar_init(&s_full[i], 1); mbar_init(&s_free[i], 128); }
+        mbar_init(&p_full, 128);
+        mbar_init(&pv_done, 1);
+        mbar_init(&drain, 1);
+        abort_flag = 0;
+        fence_barrier_init();
+        tma_prefetch_desc(&tmQ);
+        tma_prefetch_desc(&tmK);
+        tma_prefetch_desc(&tmV);
     }
+    if (warp == 2) tmem_alloc(&tmem_slot, TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+    volatile int *abort_v = &abort_flag;
 
-    float o[DH / 8][4];
-#pragma unroll
-    for (int i = 0; i < DH / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-    float m_r[2] = {-INFINITY, -INFINITY}, l_r[2] = {0.f, 0.f};
-
-    for (int kb = 0; kb < nkb; ++kb) {
-        const int buf = kb & 1;
-        if (kb + 1 < nkb) {
-            load_rows<DH>(Ks + (buf ^ 1) * KV_TILE, Kh, ldkv, (kb + 1) * BC, BC, L);
-            load_rows<DH>(Vs + (buf ^ 1) * KV_TILE, Vh, ldkv, (kb + 1) * BC, BC, L);
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer ----------------
+        const int x0 = h * DH;
+        mbar_arrive_expect_tx(&q_full, C::Q_BYTES);
+        for (int a = 0; a < C::ATOMS; ++a) tma_load_2d(Qs + a * ATOM_BYTES, &tmQ, &q_full, x0 + 64 * a, q0);
+        int k_issued = 0, v_issued = 0;
+        for (int j = 0; j < nb; ++j) {
+            const int ks = j % KST;
+            if (!mbar_wait(&k_empty[ks], ((j / KST) & 1) ^ 1, abort_v, p.err)) break;
+            mbar_arrive_expect_tx(&k_full[ks], C::K_BYTES);
+            for (int a = 0; a < C::ATOMS; ++a)
+                tma_load_2d(Ks + ks * C::K_BYTES + a * ATOM_BYTES, &tmK, &k_full[ks], x0 + 64 * a, j * BN);
+            k_issued = j + 1;
+            const int vs = j % VST;
+            if (!mbar_wait(&v_empty[vs], ((j / VST) & 1) ^ 1, abort_v, p.err)) break;
+            mbar_arrive_expect_tx(&v_full[vs], C::V_BYTES);
+            for (int a = 0; a < C::ATOMS; ++a)
+                tma_load_2d(Vs + vs * C::V_BYTES + a * ATOM_BYTES, &tmV, &v_full[vs], x0 + 64 * a, j * BN);
+            v_issued = j + 1;
         }
-        cp_async_commit();
-        const uint8_t *Kt = Ks + buf * KV_TILE;
-        const uint8_t *Vt = Vs + buf * KV_TILE;
-
-        float s[BC / 8][4];
+        if (*abort_v) {  // let this CTA's copies land before it exits
+            mbar_wait(&q_full, 0, abort_v, nullptr, 100000000ull);
+            for (int j = k_issued - KST < 0 ? 0 : k_issued - KST; j < k_issued; ++j)
+                mbar_wait(&k_full[j % KST], (j / KST) & 1, abort_v, nullptr, 100000000ull);
+            for (int j = v_issued - VST < 0 ? 0 : v_issued - VST; j < v_issued; ++j)
+                mbar_wait(&v_full[j % VST], (j / VST) & 1, abort_v, nullptr, 100000000ull);
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer ----------------
+        bool ok = mbar_wait(&q_full, 0, abort_v, p.err);
+        for (int j = 0; ok && j <= nb; ++j) {
+            if (j < nb) {
+                const int b = j & 1;
+                if (j >= 2 && !mbar_wait(&s_free[b], ((j >> 1) - 1) & 1, abort_v, p.err)) { ok = false; break; }
+                const int ks = j % KST;
+                if (!mbar_wait(&k_full[ks], (j / KST) & 1, abort_v, p.err)) { ok = false; break; }
+                tc_fence_after();
+                const uint8_t *kt = Ks + ks * C::K_BYTES;
 #pragma unroll
-        for (int nt = 0; nt < BC / 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+                for (int kk = 0; kk < DH / 16; ++kk) {
+                    const int a = kk >> 2, off = (kk & 3) * 32;
+                    tc_mma_f16(tmem + (uint32_t)(b * BN), smem_desc_sw128(Qs + a * ATOM_BYTES + off),
+                               smem_desc_sw128(kt + a * ATOM_BYTES + off), C::IDESC_S, kk > 0);
+                }
+                tc_commit(&s_full[b]);
+                tc_commit(&k_empty[ks]);
+            }
+            if (j >= 1) {
+                const int jj = j - 1;
+                if (!mbar_wait(&p_full, jj & 1, abort_v, p.err)) { ok = false; break; }
+                const int vs = jj % VST;
+                if (!mbar_wait(&v_full[vs], (jj / VST) & 1, abort_v, p.err)) { ok = false; break; }
+                tc_fence_after();
+                const uint8_t *vt = Vs + vs * C::V_BYTES;
 #pragma unroll
-        for (int np = 0; np < BC / 16; ++np) {        // pairs of 8-key tiles
-            const int kr = np * 16 + (lane & 7) + 8 * (lane >> 4);
-#pragma unroll
-            for (int ks = 0; ks < DH / 16; ++ks) {
-                uint32_t b[4];
-                ldsm_x4(b, Kt + sw<DH>(kr, ks * 2 + ((lane >> 3) & 1)));
-                mma_bf16(s[2 * np], qf[ks], b[0], b[1]);
-                mma_bf16(s[2 * np + 1], qf[ks], b[2], b[3]);
+                for (int kk = 0; kk < BN / 16; ++kk) {
+                    const int a = kk >> 2, off = (kk & 3) * 32;
+                    tc_mma_f16(tmem + O_COL, smem_desc_sw128(Ps + a * ATOM_BYTES + off),
+                               smem_desc_sw128_mn(vt + kk * 2048, ATOM_BYTES, 1024), C::IDESC_PV,
+                               (jj > 0 || kk > 0) ? 1u : 0u);
+                }
+                tc_commit(&pv_done);
+                tc_commit(&v_empty[vs]);
             }
         }
-        const int key0 = kb * BC;
-        if (key0 + BC > L) {
-#pragma unroll
-            for (int nt = 0; nt < BC / 8; ++nt) {
-                const int j = key0 + nt * 8 + 2 * (lane & 3);
-                if (j >= L) s[nt][0] = s[nt][2] = -INFINITY;
-                if (j + 1 >= L) s[nt][1] = s[nt][3] = -INFINITY;
-            }
+        if (!ok) {  // wait for the MMAs already issued before tensor memory is freed
+            tc_commit(&drain);
+            mbar_wait(&drain, 0, abort_v, nullptr, 100000000ull);
         }
-        // online softmax over the two rows this thread holds (g and g + 8)
+    } else if (warp >= 4) {
+        // ---------------- softmax / correction / epilogue ----------------
+        const int r = (warp - 4) * 32 + lane;          // row of the tile = TMEM lane
+        const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+        const float sl2 = p.scale_log2;
+        float m_used = -INFINITY, l = 0.f;
+        bool ok = true;
+        uint8_t *prow = Ps + r * 128;
+        const int sw = r & 7;
+        for (int j = 0; j < nb; ++j) {
+            const int b = j & 1;
+            ok = __all_sync(0xffffffffu, mbar_wait(&s_full[b], (j >> 1) & 1, abort_v, p.err));
+            if (!ok) break;
+            tc_fence_after();
+            uint32_t sraw[BN];
 #pragma unroll
-        for (int hr = 0; hr < 2; ++hr) {
-            float mx = -INFINITY;
+            for (int c = 0; c < BN / 32; ++c)
+                tmem_ld32(tmem + lane_base + (uint32_t)(b * BN + 32 * c), sraw + 32 * c);
+            tmem_ld_wait();
+            float s[BN];
 #pragma unroll
-            for (int nt = 0; nt < BC / 8; ++nt)
-                mx = fmaxf(mx, fmaxf(s[nt][2 * hr], s[nt][2 * hr + 1]));
-            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-            const float m_new = fmaxf(m_r[hr], mx * scale_log2);
-            const float alpha = exp2f(m_r[hr] - m_new);
+            for (int i = 0; i < BN; ++i) s[i] = __uint_as_float(sraw[i]);
+            tc_fence_before();
+            mbar_arrive(&s_free[b]);
+            const int kvalid = p.L - j * BN;                 // keys of this block that exist
+            if (kvalid < BN) {
+#pragma unroll
+                for (int i = 0; i < BN; ++i)
+                    if (i >= kvalid) s[i] = -INFINITY;
+            }
+            float mx = s[0];
+#pragma unroll
+            for (int i = 1; i < BN; ++i) mx = fmaxf(mx, s[i]);
+            const float m_new = fmaxf(m_used, mx * sl2);
+            const bool need = m_new > m_used + RESCALE_LOG2;
+            float alpha = 1.f;
+            if (need) {
+                alpha = ex2_approx(m_used - m_new);
+                l *= alpha;
+                m_used = m_new;
+            }
+            const bool warp_rescale = __any_sync(0xffffffffu, need) && j > 0;
+            uint32_t pk[BN / 2];
             float rs = 0.f;
 #pragma unroll
-            for (int nt = 0; nt < BC / 8; ++nt) {
-                const float p0 = exp2f(s[nt][2 * hr] * scale_log2 - m_new);
-                const float p1 = exp2f(s[nt][2 * hr + 1] * scale_log2 - m_new);
-                s[nt][2 * hr] = p0;
-                s[nt][2 * hr + 1] = p1;
-                rs += p0 + p1;
+            for (int i = 0; i < BN / 2; ++i) {
+                const float p0 = ex2_approx(fmaf(s[2 * i], sl2, -m_used));
+                const float p1 = ex2_approx(fmaf(s[2 * i + 1], sl2, -m_used));
+                pk[i] = pack_bf16(p0, p1);
+                rs += bf16lo(pk[i]) + bf16hi(pk[i]);
             }
-            rs += __shfl_xor_sync(0xffffffffu, rs, 1);
-            rs += __shfl_xor_sync(0xffffffffu, rs, 2);
-            l_r[hr] = l_r[hr] * alpha + rs;
-            m_r[hr] = m_new;
+            l += rs;
+            if (j >= 1) {   // P_{j-1} and O are in use by P V_{j-1} until it completes
+                ok = __all_sync(0xffffffffu, mbar_wait(&pv_done, (j - 1) & 1, abort_v, p.err));
+                if (!ok) break;
+                tc_fence_after();
+            }
 #pragma unroll
-            for (int dt = 0; dt < DH / 8; ++dt) {
-                o[dt][2 * hr] *= alpha;
-                o[dt][2 * hr + 1] *= alpha;
+            for (int a = 0; a < 2; ++a)
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    const uint32_t *src = pk + a * 32 + c * 4;
+                    *reinterpret_cast<uint4 *>(prow + a * ATOM_BYTES + ((c ^ sw) << 4)) =
+                        make_uint4(src[0], src[1], src[2], src[3]);
+                }
+            if (warp_rescale) {
+#pragma unroll
+                for (int c = 0; c < DH / 32; ++c) {
+                    uint32_t o[32];
+                    tmem_ld32(tmem + lane_base + O_COL + 32 * c, o);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+                    tmem_st32(tmem + lane_base + O_COL + 32 * c, o);
+                }
+                tmem_st_wait();
+            }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            mbar_arrive(&p_full);
+        }
+        if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&pv_done, (nb - 1) & 1, abort_v, p.err));
+        if (ok) {
+            tc_fence_after();
+            const int row = q0 + r;
+            const float inv = 1.f / l;
+            __nv_bfloat16 *dst = p.O + (int64_t)row * p.ldo + h * DH;
+#pragma unroll
+            for (int c = 0; c < DH / 32; ++c) {
+                uint32_t o[32];
+                tmem_ld32(tmem + lane_base + O_COL + 32 * c, o);
+                tmem_ld_wait();
+                if (row < p.M) {
+                    float f[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) f[i] = __uint_as_float(o[i]) * inv;
+                    uint4 *op = reinterpret_cast<uint4 *>(dst + 32 * c);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) op[i] = pack8_bf16(f + 8 * i);
+                }
             }
         }
-        // O += P V
-#pragma unroll
-        for (int ks = 0; ks < BC / 16; ++ks) {
-            uint32_t a[4];
-            a[0] = pack_bf16(s[2 * ks][0], s[2 * ks][1]);
-            a[1] = pack_bf16(s[2 * ks][2], s[2 * ks][3]);
-            a[2] = pack_bf16(s[2 * ks + 1][0], s[2 * ks + 1][1]);
-            a[3] = pack_bf16(s[2 * ks + 1][2], s[2 * ks + 1][3]);
-            const int vr = ks * 16 + (lane & 7) + 8 * ((lane >> 3) & 1);
-#pragma unroll
-            for (int dp = 0; dp < DH / 16; ++dp) {
-                uint32_t b[4];
-                ldsm_x4_t(b, Vt + sw<DH>(vr, dp * 2 + (lane >> 4)));
-                mma_bf16(o[2 * dp], a, b[0], b[1]);
-                mma_bf16(o[2 * dp + 1], a, b[2], b[3]);
-            }
-        }
-        cp_async_wait_all();
-        __syncthreads();
     }
-
-    // normalise and store
-    const int g = lane >> 2, t = lane & 3;
-#pragma unroll
-    for (int hr = 0; hr < 2; ++hr) {
-        const int row = q0 + warp * 16 + g + 8 * hr;
-        if (row >= M) continue;
-        const float inv = 1.f / l_r[hr];
-        __nv_bfloat16 *dst = O + (int64_t)row * ldo + h * DH;
-#pragma unroll
-        for (int dt = 0; dt < DH / 8; ++dt) {
-            const uint32_t v = pack_bf16(o[dt][2 * hr] * inv, o[dt][2 * hr + 1] * inv);
-            *reinterpret_cast<uint32_t *>(dst + dt * 8 + 2 * t) = v;
-        }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 2) {
+        tc_fence_after();
+        tmem_dealloc(tmem, TMEM_COLS);
     }
 }
 
 template <int DH>
-void launch_dh(const void *Q, int64_t ldq, const void *K, const void *V, int64_t ldkv, int M, int L,
-               int H, void *O, int64_t ldo, cudaStream_t st) {
-    const size_t smem = (size_t)(BR + 4 * BC) * DH * 2;
+echo_status launch_dh(const void *Q, int64_t ldq, const void *K, const void *V, int64_t ldkv, int M,
+                      int L, int H, void *O, int64_t ldo, cudaStream_t st) {
     static int attr_done[64] = {};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-        cudaFuncSetAttribute(attn_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaFuncSetAttribute(attn_tc_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             Cfg<DH>::SMEM);
         attr_done[dev] = 1;
     }
-    dim3 grid((M + BR - 1) / BR, H);
-    const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
+    CUtensorMap tq, tk, tv;
+    const uint64_t cols = (uint64_t)H * DH;
+    if (!echo::make_tmap_bf16(&tq, Q, (uint64_t)M, cols, (uint64_t)ldq, BM) ||
+        !echo::make_tmap_bf16(&tk, K, (uint64_t)L, cols, (uint64_t)ldkv, BN) ||
+        !echo::make_tmap_bf16(&tv, V, (uint64_t)L, cols, (uint64_t)ldkv, BN))
+        return ECHO_ERR_CUDA;
+    AttnParams p;
+    p.M = M;
+    p.L = L;
+    p.scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
+    p.O = static_cast<__nv_bfloat16 *>(O);
+    p.ldo = ldo;
+    p.err = echo::device_error_ptr();
+    dim3 grid((M + BM - 1) / BM, H);
     echo::LaunchScope ls(ECHO_K_ATTENTION, M, L, (int64_t)H * DH, st);
-    attn_kernel<DH><<<grid, THREADS, smem, st>>>(
-        static_cast<const __nv_bfloat16 *>(Q), ldq, static_cast<const __nv_bfloat16 *>(K),
-        static_cast<const __nv_bfloat16 *>(V), ldkv, M, L, static_cast<__nv_bfloat16 *>(O), ldo,
-        scale_log2);
+    attn_tc_kernel<DH><<<grid, THREADS, Cfg<DH>::SMEM, st>>>(tq, tk, tv, p);
+    return echo::last_launch_status();
 }
 
 }  // namespace
 
 namespace echo {
 
-void launch_attention(const void *Q, int64_t ldq, const void *K, const void *V, int64_t ldkv,
-                      int32_t M, int32_t L, int32_t H, int32_t d, void *O, int64_t ldo,
-                      cudaStream_t st) {
-    if (M <= 0) return;
-    if (d == 64)
-        launch_dh<64>(Q, ldq, K, V, ldkv, M, L, H, O, ldo, st);
-    else
-        launch_dh<128>(Q, ldq, K, V, ldkv, M, L, H, O, ldo, st);
+echo_status launch_attention(const void *Q, int64_t ldq, const void *K, const void *V, int64_t ldkv,
+                             int32_t M, int32_t L, int32_t H, int32_t d, void *O, int64_t ldo,
+                             cudaStream_t st) {
+    if (M <= 0) return ECHO_OK;
+    if (d == 64) return launch_dh<64>(Q, ldq, K, V, ldkv, M, L, H, O, ldo, st);
+    return launch_dh<128>(Q, ldq, K, V, ldkv, M, L, H, O, ldo, st);
 }
 
 }  // namespace echo
@@ -253,6 +334,6 @@ extern "C" echo_status echo_attention(const void *Q, int64_t ldq, const void *K,
     if (!Q || !K || !V || !O) return ECHO_ERR_INVALID_ARG;
     if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O)) return ECHO_ERR_INVALID_ARG;
     if (!device_supported()) return ECHO_ERR_UNSUPPORTED;
-    launch_attention(Q, ldq, K, V, ldkv, M, L, H, d, O, ldo, reinterpret_cast<cudaStream_t>(stream));
-    return last_launch_status();
+    return launch_attention(Q, ldq, K, V, ldkv, M, L, H, d, O, ldo,
+                            reinterpret_cast<cudaStream_t>(stream));
 }

@@ -111,14 +111,16 @@ extern "C" echo_status echo_block_step(const echo_block_weights *w, const echo_b
         s = launch_linear({na, D, K, D, w->Wq, w->bq, D, 0, nullptr, ECHO_BF16, nullptr, qa, D,
                            ECHO_BF16}, st);
         if (s != ECHO_OK) return s;
-        launch_attention(qa, D, kvb, kvb + D, 2 * (int64_t)D, K, NT, d.H, d.d, att, D, st);
+        s = launch_attention(qa, D, kvb, kvb + D, 2 * (int64_t)D, K, NT, d.H, d.d, att, D, st);
+        if (s != ECHO_OK) return s;
         s = launch_linear({att, D, K, D, w->Wo, w->bo, D, 0, x, ECHO_BF16, idx, h1, D, ECHO_F32}, st);
         if (s != ECHO_OK) return s;
         launch_layernorm(h1, ECHO_F32, nullptr, K, D, na, st);
         s = launch_linear({na, D, K, D, w->Wqc, w->bqc, D, 0, nullptr, ECHO_BF16, nullptr, qa, D,
                            ECHO_BF16}, st);
         if (s != ECHO_OK) return s;
-        launch_attention(qa, D, kvc, kvc + D, 2 * (int64_t)D, K, d.Lc, d.H, d.d, att, D, st);
+        s = launch_attention(qa, D, kvc, kvc + D, 2 * (int64_t)D, K, d.Lc, d.H, d.d, att, D, st);
+        if (s != ECHO_OK) return s;
         s = launch_linear({att, D, K, D, w->Woc, w->boc, D, 0, h1, ECHO_F32, nullptr, h2, D,
                            ECHO_F32}, st);
         if (s != ECHO_OK) return s;

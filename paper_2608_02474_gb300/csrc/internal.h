@@ -54,9 +54,9 @@ struct LinearArgs {
 echo_status launch_linear(const LinearArgs &a, cudaStream_t st);
 
 // attention.cu
-void launch_attention(const void *Q, int64_t ldq, const void *K, const void *V, int64_t ldkv,
-                      int32_t M, int32_t L, int32_t H, int32_t d, void *O, int64_t ldo,
-                      cudaStream_t st);
+echo_status launch_attention(const void *Q, int64_t ldq, const void *K, const void *V, int64_t ldkv,
+                             int32_t M, int32_t L, int32_t H, int32_t d, void *O, int64_t ldo,
+                             cudaStream_t st);
 
 // cache.cu
 void launch_quant(const void *src, echo_dtype st_t, const int32_t *rows, int32_t n_rows,
