@@ -2,13 +2,15 @@
 // projections, FFN on the active latents; Sec. 3.3) on the 5th-generation
 // tensor cores:  out = act(A W^T + bias) + resid.
 //
-// One CTA per 128 x 256 output tile, 8 warps:
+// Persistent: one CTA per SM walks 128 x 256 output tiles in a banded order;
+// 8 warps:
 //   warp 0      TMA producer: A [128 x 64] and W [256 x 64] bf16 tiles, 128-byte
 //               swizzle, into a 4-stage shared-memory ring (48 KB per stage);
-//   warp 1      one elected thread issues tcgen05.mma (M=128, N=256, K=16) into a
-//               128 x 256 fp32 accumulator in tensor memory, and commits each
-//               stage back to the producer;
-//   warp 2      allocates / frees the 256 tensor-memory columns;
+//   warp 1      one thread issues tcgen05.mma (M=128, N=256, K=16) into one of two
+//               128 x 256 fp32 accumulators in tensor memory, and commits each
+//               stage back to the producer, so the epilogue of one tile overlaps
+//               the main loop of the next;
+//   warp 2      allocates / frees the 512 tensor-memory columns;
 //   warps 4..7  epilogue: tcgen05.ld 32 columns at a time (warp w reads TMEM
 //               lanes 32 (w mod 4) ..), adds bias, GELU, residual, stores.
 // Every mbarrier wait is bounded (ECHO_ERR_TIMEOUT) and a CTA that gives up
@@ -24,7 +26,8 @@ constexpr int B_BYTES = BN * BK * 2;   // 32 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024;  // + alignment slack
 constexpr int THREADS = 256;
-constexpr uint32_t TMEM_COLS = 256;
+constexpr uint32_t TMEM_COLS = 512;   // two 256-column accumulators
+constexpr int GROUP_N = 16;            // N tiles per raster band
 constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
 
 enum : int { EPI_GELU = 1, EPI_RES_BF16 = 2, EPI_RES_F32 = 4, EPI_OUT_F32 = 8 };
@@ -45,6 +48,18 @@ ECHO_DEV float gelu_tanh(float x) {
     return 0.5f * x * (1.f + tanhf(u));
 }
 
+// Tile order: bands of GROUP_N N-tiles; inside a band M is swept with the band's
+// N-tiles adjacent, so the CTAs in flight share a few A row blocks and one band
+// of W, which stay in L2 while the band is processed.
+ECHO_DEV void tile_coords(int t, int num_m, int num_n, int &mt, int &nt) {
+    const int band = t / (GROUP_N * num_m);
+    const int first_n = band * GROUP_N;
+    const int gn = min(GROUP_N, num_n - first_n);
+    const int r = t - band * GROUP_N * num_m;
+    mt = r / gn;
+    nt = first_n + r % gn;
+}
+
 template <int EPI>
 __global__ void __launch_bounds__(THREADS, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -52,20 +67,25 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                 ~static_cast<uintptr_t>(1023));
-    __shared__ __align__(8) uint64_t full_bar[STAGES], empty_bar[STAGES], accum_bar, drain_bar;
+    __shared__ __align__(8) uint64_t full_bar[STAGES], empty_bar[STAGES];
+    __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2], drain_bar;
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_flag;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM;
     const int num_kb = p.Kd / BK;
+    const int num_m = (p.M + BM - 1) / BM, num_n = (p.N + BN - 1) / BN;
+    const int num_tiles = num_m * num_n;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&full_bar[s], 1);
             mbar_init(&empty_bar[s], 1);
         }
-        mbar_init(&accum_bar, 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], 128);
+        }
         mbar_init(&drain_bar, 1);
         abort_flag = 0;
         fence_barrier_init();
@@ -81,54 +101,75 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
 
     if (warp == 0 && lane == 0) {
         // ---------------- TMA producer ----------------
-        int issued = 0;
-        for (int kb = 0; kb < num_kb; ++kb) {
-            const int s = kb % STAGES;
-            const uint32_t ph = (kb / STAGES) & 1;
-            if (!mbar_wait(&empty_bar[s], ph ^ 1, abort_v, p.err)) break;
-            uint8_t *a = smem + s * STAGE_BYTES;
-            uint8_t *b = a + A_BYTES;
-            mbar_arrive_expect_tx(&full_bar[s], STAGE_BYTES);
-            tma_load_2d(a, &tmA, &full_bar[s], kb * BK, m0);
-            tma_load_2d(b, &tmB, &full_bar[s], kb * BK, n0);
-            issued = kb + 1;
+        int it = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; ok && t < num_tiles; t += gridDim.x) {
+            int mt, nt;
+            tile_coords(t, num_m, num_n, mt, nt);
+            for (int kb = 0; kb < num_kb; ++kb, ++it) {
+                const int s = it % STAGES;
+                if (!mbar_wait(&empty_bar[s], ((it / STAGES) & 1) ^ 1, abort_v, p.err)) {
+                    ok = false;
+                    break;
+                }
+                uint8_t *a = smem + s * STAGE_BYTES;
+                mbar_arrive_expect_tx(&full_bar[s], STAGE_BYTES);
+                tma_load_2d(a, &tmA, &full_bar[s], kb * BK, mt * BM);
+                tma_load_2d(a + A_BYTES, &tmB, &full_bar[s], kb * BK, nt * BN);
+            }
         }
         if (*abort_v) {  // let this CTA's copies land before it exits
-            for (int kb = issued - STAGES < 0 ? 0 : issued - STAGES; kb < issued; ++kb)
-                mbar_wait(&full_bar[kb % STAGES], (kb / STAGES) & 1, abort_v, nullptr, 100000000ull);
+            for (int k = it - STAGES < 0 ? 0 : it - STAGES; k < it; ++k)
+                mbar_wait(&full_bar[k % STAGES], (k / STAGES) & 1, abort_v, nullptr, 100000000ull);
         }
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer ----------------
         bool ok = true;
-        for (int kb = 0; kb < num_kb; ++kb) {
-            const int s = kb % STAGES;
-            const uint32_t ph = (kb / STAGES) & 1;
-            if (!mbar_wait(&full_bar[s], ph, abort_v, p.err)) { ok = false; break; }
-            tc_fence_after();
-            const uint8_t *a = smem + s * STAGE_BYTES;
-            const uint8_t *b = a + A_BYTES;
-#pragma unroll
-            for (int k = 0; k < BK / 16; ++k) {
-                const uint64_t ad = smem_desc_sw128(a + k * 32);
-                const uint64_t bd = smem_desc_sw128(b + k * 32);
-                tc_mma_f16(tmem, ad, bd, IDESC, (kb | k) != 0);
+        int it = 0, local = 0;
+        for (int t = blockIdx.x; ok && t < num_tiles; t += gridDim.x, ++local) {
+            const int buf = local & 1;
+            if (!mbar_wait(&acc_empty[buf], ((local >> 1) & 1) ^ 1, abort_v, p.err)) {
+                ok = false;
+                break;
             }
-            tc_commit(&empty_bar[s]);
+            tc_fence_after();
+            const uint32_t d_tmem = tmem + (uint32_t)(buf * BN);
+            for (int kb = 0; kb < num_kb; ++kb, ++it) {
+                const int s = it % STAGES;
+                if (!mbar_wait(&full_bar[s], (it / STAGES) & 1, abort_v, p.err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint8_t *a = smem + s * STAGE_BYTES;
+                const uint8_t *b = a + A_BYTES;
+#pragma unroll
+                for (int k = 0; k < BK / 16; ++k)
+                    tc_mma_f16(d_tmem, smem_desc_sw128(a + k * 32), smem_desc_sw128(b + k * 32), IDESC,
+                               (kb | k) != 0);
+                tc_commit(&empty_bar[s]);
+            }
+            if (ok) tc_commit(&acc_full[buf]);
         }
-        if (ok) {
-            tc_commit(&accum_bar);
-        } else {  // wait for the MMAs already issued before tensor memory is freed
+        if (!ok) {  // wait for the MMAs already issued before tensor memory is freed
             tc_commit(&drain_bar);
             mbar_wait(&drain_bar, 0, abort_v, nullptr, 100000000ull);
         }
     } else if (warp >= 4) {
         // ---------------- epilogue ----------------
         const int q = warp & 3;
-        const bool ok = __all_sync(0xffffffffu, mbar_wait(&accum_bar, 0, abort_v, p.err,
-                                                          4000000000ull));
-        tc_fence_after();
-        if (ok) {
-            const int row = m0 + q * 32 + lane;
+        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+        int local = 0;
+        for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++local) {
+            const int buf = local & 1;
+            const bool ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[buf], (local >> 1) & 1,
+                                                              abort_v, p.err, 4000000000ull));
+            if (!ok) break;
+            tc_fence_after();
+            int mt, nt;
+            tile_coords(t, num_m, num_n, mt, nt);
+            const int n0 = nt * BN;
+            const int row = mt * BM + q * 32 + lane;
             const bool row_ok = row < p.M;
             int rrow = row;
             if ((EPI & EPI_RES_BF16) && p.resid_rows && row_ok) rrow = p.resid_rows[row];
@@ -136,7 +177,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                 const int col = n0 + c;
                 if (col >= p.N) break;                       // warp-uniform
                 uint32_t r[32];
-                tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c, r);
+                tmem_ld32(tmem + lane_base + (uint32_t)(buf * BN + c), r);
                 tmem_ld_wait();
                 if (!row_ok) continue;
                 float v[32];
@@ -159,10 +200,10 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                         static_cast<const __nv_bfloat16 *>(p.resid) + (int64_t)rrow * p.N + col);
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {
-                        float t[8];
-                        unpack8_bf16(__ldg(rp + i), t);
+                        float tt[8];
+                        unpack8_bf16(__ldg(rp + i), tt);
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) v[8 * i + e] += t[e];
+                        for (int e = 0; e < 8; ++e) v[8 * i + e] += tt[e];
                     }
                 }
                 if (EPI & EPI_RES_F32) {
@@ -170,8 +211,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                         static_cast<const float *>(p.resid) + (int64_t)row * p.N + col);
 #pragma unroll
                     for (int i = 0; i < 8; ++i) {
-                        const float4 t = __ldg(rp + i);
-                        v[4 * i] += t.x; v[4 * i + 1] += t.y; v[4 * i + 2] += t.z; v[4 * i + 3] += t.w;
+                        const float4 tt = __ldg(rp + i);
+                        v[4 * i] += tt.x; v[4 * i + 1] += tt.y; v[4 * i + 2] += tt.z; v[4 * i + 3] += tt.w;
                     }
                 }
                 if (EPI & EPI_OUT_F32) {
@@ -187,6 +228,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                     for (int i = 0; i < 4; ++i) op[i] = pack8_bf16(v + 8 * i);
                 }
             }
+            tc_fence_before();
+            mbar_arrive(&acc_empty[buf]);
         }
     }
     tc_fence_before();
@@ -195,6 +238,18 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
         tc_fence_after();
         tmem_dealloc(tmem, TMEM_COLS);
     }
+}
+
+int num_sms() {
+    static int cached[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+    if (!cached[dev]) {
+        int n = 0;
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        cached[dev] = n > 0 ? n : 1;
+    }
+    return cached[dev];
 }
 
 template <int EPI>
@@ -208,7 +263,8 @@ echo_status run(const CUtensorMap &ta, const CUtensorMap &tb, const GemmParams &
             return ECHO_ERR_CUDA;
         attr_set[dev] = 1;
     }
-    dim3 grid((p.N + BN - 1) / BN, (p.M + BM - 1) / BM);
+    const int tiles = ((p.M + BM - 1) / BM) * ((p.N + BN - 1) / BN);
+    const int grid = tiles < num_sms() ? tiles : num_sms();
     echo::LaunchScope ls(ECHO_K_GEMM, p.M, p.N, p.Kd, st);
     gemm_kernel<EPI><<<grid, THREADS, SMEM_BYTES, st>>>(ta, tb, p);
     return echo::last_launch_status();
