@@ -3,20 +3,23 @@
 // audio condition tokens (cross-attention).
 //
 // Flash-style forward on the 5th-generation tensor cores.  One CTA per
-// (128-query tile, head), 8 warps:
-//   warp 0      TMA producer: the Q tile once, then 128-key blocks of K and V
-//               (128-byte swizzle, 64-column boxes) into two-stage rings;
-//   warp 1      one thread issues S_j = Q K_j^T (M 128, N 128, K d) into one of
-//               two TMEM S buffers, and O += P_j V_j (M 128, N d, K 128; V is
-//               read MN-major straight from its row-major tile) into a TMEM O
-//               accumulator, one block behind;
-//   warp 2      allocates / frees 512 TMEM columns (S0, S1, O);
-//   warps 4..7  softmax, one query row per thread (its TMEM lane): tcgen05.ld of
-//               the S row, online max, P = 2^(s*scale - m) rounded to bf16 into a
-//               swizzled shared-memory tile (the A operand of P V), row sum of the
-//               rounded P; O is rescaled in TMEM only when the running max grows
-//               by more than 2^8 (otherwise the stale max is kept, which is exact
-//               after the final division by the row sum); final O / l to bf16.
+// (two 128-query tiles, head), 12 warps, with the two tiles in ping-pong so
+// that one tile's softmax runs while the tensor cores work on the other:
+//   warp 0      TMA producer: both Q tiles once, then 128-key blocks K_0, V_0,
+//               K_1, V_1, ... (128-byte swizzle, 64-column boxes) into a
+//               three-slot ring shared by K and V;
+//   warp 1      one thread issues S_t = Q_t K_j^T (M 128, N 128, K d) into the
+//               tile's TMEM S buffer and O_t += P_t V_j (M 128, N d, K 128; V is
+//               read MN-major straight from its row-major tile) into the tile's
+//               TMEM O accumulator, in the order PV0_j S0_{j+1} PV1_j S1_{j+1};
+//   warp 2      allocates / frees 512 TMEM columns (S0, S1, O0, O1);
+//   warps 4..7  softmax of tile 0, warps 8..11 softmax of tile 1, one query row
+//               per thread (its TMEM lane): tcgen05.ld of the S row, online max,
+//               P = 2^(s*scale - m) rounded to bf16 into the tile's swizzled
+//               shared-memory P buffer (the A operand of P V), row sum of P; O is
+//               rescaled in TMEM only when the running max grows by more than
+//               2^8 (otherwise the stale max is kept, which is exact after the
+//               final division by the row sum); final O / l to bf16.
 // Keys beyond L are masked to P = 0; queries beyond M run on zero rows and are
 // not stored.  Every mbarrier wait is bounded (ECHO_ERR_TIMEOUT).
 #include "common.cuh"
@@ -24,12 +27,12 @@
 
 namespace {
 
-constexpr int BM = 128;        // queries per CTA
+constexpr int BM = 128;        // queries per tile; two tiles per CTA
+constexpr int TILES = 2;
 constexpr int BN = 128;        // keys per block
-constexpr int KST = 2;         // K ring stages
-constexpr int VST = 2;         // V ring stages
-constexpr int THREADS = 256;
-constexpr uint32_t TMEM_COLS = 512;
+constexpr int RING = 3;        // K/V ring slots (K_j and V_j alternate)
+constexpr int THREADS = 384;   // 4 control warps + 2 softmax warpgroups
+constexpr uint32_t TMEM_COLS = 512;   // S0, S1, O0, O1
 constexpr uint32_t O_COL = 256;
 constexpr int ATOM_BYTES = 128 * 128;   // one [128 rows x 64 bf16] 128B-swizzled box
 constexpr float RESCALE_LOG2 = 8.f;
@@ -38,10 +41,9 @@ template <int DH>
 struct Cfg {
     static constexpr int ATOMS = DH / 64;
     static constexpr int Q_BYTES = BM * DH * 2;
-    static constexpr int K_BYTES = BN * DH * 2;
-    static constexpr int V_BYTES = BN * DH * 2;
+    static constexpr int SLOT_BYTES = BN * DH * 2;
     static constexpr int P_BYTES = BM * BN * 2;
-    static constexpr int SMEM = Q_BYTES + KST * K_BYTES + VST * V_BYTES + P_BYTES + 1024;
+    static constexpr int SMEM = TILES * Q_BYTES + RING * SLOT_BYTES + TILES * P_BYTES + 1024;
     static constexpr uint32_t IDESC_S = idesc_bf16_f32(BM, BN);
     static constexpr uint32_t IDESC_PV = idesc_bf16_f32(BM, DH) | (1u << 16);  // B MN-major
 };
@@ -62,28 +64,32 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                 ~static_cast<uintptr_t>(1023));
-    uint8_t *Qs = smem;
-    uint8_t *Ks = Qs + C::Q_BYTES;
-    uint8_t *Vs = Ks + KST * C::K_BYTES;
-    uint8_t *Ps = Vs + VST * C::V_BYTES;
+    uint8_t *Qs = smem;                                  // [TILES][Q_BYTES]
+    uint8_t *Ring = Qs + TILES * C::Q_BYTES;             // [RING][SLOT_BYTES]
+    uint8_t *Ps = Ring + RING * C::SLOT_BYTES;           // [TILES][P_BYTES]
 
-    __shared__ __align__(8) uint64_t q_full, k_full[KST], k_empty[KST], v_full[VST], v_empty[VST];
-    __shared__ __align__(8) uint64_t s_full[2], s_free[2], p_full, pv_done, drain;
+    // Every barrier is reused only after its previous phase has been observed
+    // by its waiter, so no waiter can fall two phases behind.
+    __shared__ __align__(8) uint64_t q_full, ring_full[RING], ring_empty[RING];
+    __shared__ __align__(8) uint64_t s_full[TILES], s_free[TILES], p_full[TILES], pv_done[TILES];
+    __shared__ __align__(8) uint64_t drain;
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_flag;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int h = blockIdx.y;
-    const int q0 = blockIdx.x * BM;
+    const int q0 = blockIdx.x * (TILES * BM);
     const int nb = (p.L + BN - 1) / BN;
 
     if (threadIdx.x == 0) {
         mbar_init(&q_full, 1);
-        for (int i = 0; i < KST; ++i) { mbar_init(&k_full[i], 1); mbar_init(&k_empty[i], 1); }
-        for (int i = 0; i < VST; ++i) { mbar_init(&v_full[i], 1); mbar_init(&v_empty[i], 1); }
-        for (int i = 0; i < 2; ++i) { mbar_init(&s_full[i], 1); mbar_init(&s_free[i], 128); }
-        mbar_init(&p_full, 128);
-        mbar_init(&pv_done, 1);
+        for (int i = 0; i < RING; ++i) { mbar_init(&ring_full[i], 1); mbar_init(&ring_empty[i], 1); }
+        for (int t = 0; t < TILES; ++t) {
+            mbar_init(&s_full[t], 1);
+            mbar_init(&s_free[t], 4);    // one arrival per softmax warp
+            mbar_init(&p_full[t], 4);
+            mbar_init(&pv_done[t], 1);
+        }
         mbar_init(&drain, 1);
         abort_flag = 0;
         fence_barrier_init();
@@ -99,68 +105,73 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     volatile int *abort_v = &abort_flag;
 
     if (warp == 0 && lane == 0) {
-        // ---------------- TMA producer ----------------
+        // ---------------- TMA producer: Q0, Q1, then K_0, V_0, K_1, V_1, ... ----------------
         const int x0 = h * DH;
-        mbar_arrive_expect_tx(&q_full, C::Q_BYTES);
-        for (int a = 0; a < C::ATOMS; ++a) tma_load_2d(Qs + a * ATOM_BYTES, &tmQ, &q_full, x0 + 64 * a, q0);
-        int k_issued = 0, v_issued = 0;
-        for (int j = 0; j < nb; ++j) {
-            const int ks = j % KST;
-            if (!mbar_wait(&k_empty[ks], ((j / KST) & 1) ^ 1, abort_v, p.err)) break;
-            mbar_arrive_expect_tx(&k_full[ks], C::K_BYTES);
+        mbar_arrive_expect_tx(&q_full, TILES * C::Q_BYTES);
+        for (int t = 0; t < TILES; ++t)
             for (int a = 0; a < C::ATOMS; ++a)
-                tma_load_2d(Ks + ks * C::K_BYTES + a * ATOM_BYTES, &tmK, &k_full[ks], x0 + 64 * a, j * BN);
-            k_issued = j + 1;
-            const int vs = j % VST;
-            if (!mbar_wait(&v_empty[vs], ((j / VST) & 1) ^ 1, abort_v, p.err)) break;
-            mbar_arrive_expect_tx(&v_full[vs], C::V_BYTES);
+                tma_load_2d(Qs + t * C::Q_BYTES + a * ATOM_BYTES, &tmQ, &q_full, x0 + 64 * a,
+                            q0 + t * BM);
+        int issued = 0;
+        for (int li = 0; li < 2 * nb; ++li) {
+            const int slot = li % RING;
+            if (!mbar_wait(&ring_empty[slot], ((li / RING) & 1) ^ 1, abort_v, p.err)) break;
+            mbar_arrive_expect_tx(&ring_full[slot], C::SLOT_BYTES);
+            const CUtensorMap *m = (li & 1) ? &tmV : &tmK;
             for (int a = 0; a < C::ATOMS; ++a)
-                tma_load_2d(Vs + vs * C::V_BYTES + a * ATOM_BYTES, &tmV, &v_full[vs], x0 + 64 * a, j * BN);
-            v_issued = j + 1;
+                tma_load_2d(Ring + slot * C::SLOT_BYTES + a * ATOM_BYTES, m, &ring_full[slot],
+                            x0 + 64 * a, (li >> 1) * BN);
+            issued = li + 1;
         }
         if (*abort_v) {  // let this CTA's copies land before it exits
             mbar_wait(&q_full, 0, abort_v, nullptr, 100000000ull);
-            for (int j = k_issued - KST < 0 ? 0 : k_issued - KST; j < k_issued; ++j)
-                mbar_wait(&k_full[j % KST], (j / KST) & 1, abort_v, nullptr, 100000000ull);
-            for (int j = v_issued - VST < 0 ? 0 : v_issued - VST; j < v_issued; ++j)
-                mbar_wait(&v_full[j % VST], (j / VST) & 1, abort_v, nullptr, 100000000ull);
+            for (int li = issued - RING < 0 ? 0 : issued - RING; li < issued; ++li)
+                mbar_wait(&ring_full[li % RING], (li / RING) & 1, abort_v, nullptr, 100000000ull);
         }
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer ----------------
+        // order: S0_0 S1_0 | PV0_0 S0_1 PV1_0 S1_1 | PV0_1 S0_2 PV1_1 S1_2 | ...
         bool ok = mbar_wait(&q_full, 0, abort_v, p.err);
-        for (int j = 0; ok && j <= nb; ++j) {
-            if (j < nb) {
-                const int b = j & 1;
-                if (j >= 2 && !mbar_wait(&s_free[b], ((j >> 1) - 1) & 1, abort_v, p.err)) { ok = false; break; }
-                const int ks = j % KST;
-                if (!mbar_wait(&k_full[ks], (j / KST) & 1, abort_v, p.err)) { ok = false; break; }
-                tc_fence_after();
-                const uint8_t *kt = Ks + ks * C::K_BYTES;
+        auto issue_s = [&](int t, int j) -> bool {
+            const int li = 2 * j, slot = li % RING;
+            if (j > 0 && !mbar_wait(&s_free[t], (j - 1) & 1, abort_v, p.err)) return false;
+            if (!mbar_wait(&ring_full[slot], (li / RING) & 1, abort_v, p.err)) return false;
+            tc_fence_after();
+            const uint8_t *qt = Qs + t * C::Q_BYTES;
+            const uint8_t *kt = Ring + slot * C::SLOT_BYTES;
 #pragma unroll
-                for (int kk = 0; kk < DH / 16; ++kk) {
-                    const int a = kk >> 2, off = (kk & 3) * 32;
-                    tc_mma_f16(tmem + (uint32_t)(b * BN), smem_desc_sw128(Qs + a * ATOM_BYTES + off),
-                               smem_desc_sw128(kt + a * ATOM_BYTES + off), C::IDESC_S, kk > 0);
-                }
-                tc_commit(&s_full[b]);
-                tc_commit(&k_empty[ks]);
+            for (int kk = 0; kk < DH / 16; ++kk) {
+                const int a = kk >> 2, off = (kk & 3) * 32;
+                tc_mma_f16(tmem + (uint32_t)(t * BN), smem_desc_sw128(qt + a * ATOM_BYTES + off),
+                           smem_desc_sw128(kt + a * ATOM_BYTES + off), C::IDESC_S, kk > 0);
             }
-            if (j >= 1) {
-                const int jj = j - 1;
-                if (!mbar_wait(&p_full, jj & 1, abort_v, p.err)) { ok = false; break; }
-                const int vs = jj % VST;
-                if (!mbar_wait(&v_full[vs], (jj / VST) & 1, abort_v, p.err)) { ok = false; break; }
-                tc_fence_after();
-                const uint8_t *vt = Vs + vs * C::V_BYTES;
+            tc_commit(&s_full[t]);
+            if (t == TILES - 1) tc_commit(&ring_empty[slot]);   // K_j no longer needed
+            return true;
+        };
+        auto issue_pv = [&](int t, int j) -> bool {
+            const int li = 2 * j + 1, slot = li % RING;
+            if (!mbar_wait(&p_full[t], j & 1, abort_v, p.err)) return false;
+            if (!mbar_wait(&ring_full[slot], (li / RING) & 1, abort_v, p.err)) return false;
+            tc_fence_after();
+            const uint8_t *pt = Ps + t * C::P_BYTES;
+            const uint8_t *vt = Ring + slot * C::SLOT_BYTES;
 #pragma unroll
-                for (int kk = 0; kk < BN / 16; ++kk) {
-                    const int a = kk >> 2, off = (kk & 3) * 32;
-                    tc_mma_f16(tmem + O_COL, smem_desc_sw128(Ps + a * ATOM_BYTES + off),
-                               smem_desc_sw128_mn(vt + kk * 2048, ATOM_BYTES, 1024), C::IDESC_PV,
-                               (jj > 0 || kk > 0) ? 1u : 0u);
-                }
-                tc_commit(&pv_done);
-                tc_commit(&v_empty[vs]);
+            for (int kk = 0; kk < BN / 16; ++kk) {
+                const int a = kk >> 2, off = (kk & 3) * 32;
+                tc_mma_f16(tmem + O_COL + (uint32_t)(t * DH), smem_desc_sw128(pt + a * ATOM_BYTES + off),
+                           smem_desc_sw128_mn(vt + kk * 2048, ATOM_BYTES, 1024), C::IDESC_PV,
+                           (j > 0 || kk > 0) ? 1u : 0u);
+            }
+            tc_commit(&pv_done[t]);
+            if (t == TILES - 1) tc_commit(&ring_empty[slot]);   // V_j no longer needed
+            return true;
+        };
+        for (int t = 0; ok && t < TILES; ++t) ok = issue_s(t, 0);
+        for (int j = 0; ok && j < nb; ++j) {
+            for (int t = 0; ok && t < TILES; ++t) {
+                ok = issue_pv(t, j);
+                if (ok && j + 1 < nb) ok = issue_s(t, j + 1);
             }
         }
         if (!ok) {  // wait for the MMAs already issued before tensor memory is freed
@@ -168,38 +179,48 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             mbar_wait(&drain, 0, abort_v, nullptr, 100000000ull);
         }
     } else if (warp >= 4) {
-        // ---------------- softmax / correction / epilogue ----------------
-        const int r = (warp - 4) * 32 + lane;          // row of the tile = TMEM lane
-        const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+        // ---------------- softmax / correction / epilogue of tile t ----------------
+        const int t = (warp - 4) >> 2;
+        const int quad = warp & 3;
+        const int r = quad * 32 + lane;                // row of the tile = TMEM lane
+        const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+        const uint32_t s_col = (uint32_t)(t * BN);
+        const uint32_t o_col = O_COL + (uint32_t)(t * DH);
         const float sl2 = p.scale_log2;
         float m_used = -INFINITY, l = 0.f;
         bool ok = true;
-        uint8_t *prow = Ps + r * 128;
+        uint8_t *prow = Ps + t * C::P_BYTES + r * 128;
         const int sw = r & 7;
         for (int j = 0; j < nb; ++j) {
-            const int b = j & 1;
-            ok = __all_sync(0xffffffffu, mbar_wait(&s_full[b], (j >> 1) & 1, abort_v, p.err));
+            ok = __all_sync(0xffffffffu, mbar_wait(&s_full[t], j & 1, abort_v, p.err));
             if (!ok) break;
             tc_fence_after();
-            uint32_t sraw[BN];
-#pragma unroll
-            for (int c = 0; c < BN / 32; ++c)
-                tmem_ld32(tmem + lane_base + (uint32_t)(b * BN + 32 * c), sraw + 32 * c);
-            tmem_ld_wait();
-            float s[BN];
-#pragma unroll
-            for (int i = 0; i < BN; ++i) s[i] = __uint_as_float(sraw[i]);
-            tc_fence_before();
-            mbar_arrive(&s_free[b]);
+            // pass 1: row max over the 128 keys of the block (3-input max)
             const int kvalid = p.L - j * BN;                 // keys of this block that exist
-            if (kvalid < BN) {
+            float mx;
+            {
+                float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-                for (int i = 0; i < BN; ++i)
-                    if (i >= kvalid) s[i] = -INFINITY;
+                for (int c = 0; c < BN / 64; ++c) {
+                    float sv[64];
+                    tmem_ld32(tmem + lane_base + s_col + 64 * c, reinterpret_cast<uint32_t *>(sv));
+                    tmem_ld32(tmem + lane_base + s_col + 64 * c + 32, reinterpret_cast<uint32_t *>(sv + 32));
+                    tmem_ld_wait();
+                    if (kvalid < 64 * (c + 1)) {                 // tail block only
+#pragma unroll
+                        for (int i = 0; i < 64; ++i)
+                            if (64 * c + i >= kvalid) sv[i] = -INFINITY;
+                    }
+#pragma unroll
+                    for (int i = 0; i < 64; i += 8) {
+                        m4[0] = fmax3(m4[0], sv[i], sv[i + 1]);
+                        m4[1] = fmax3(m4[1], sv[i + 2], sv[i + 3]);
+                        m4[2] = fmax3(m4[2], sv[i + 4], sv[i + 5]);
+                        m4[3] = fmax3(m4[3], sv[i + 6], sv[i + 7]);
+                    }
+                }
+                mx = fmaxf(fmax3(m4[0], m4[1], m4[2]), m4[3]);
             }
-            float mx = s[0];
-#pragma unroll
-            for (int i = 1; i < BN; ++i) mx = fmaxf(mx, s[i]);
             const float m_new = fmaxf(m_used, mx * sl2);
             const bool need = m_new > m_used + RESCALE_LOG2;
             float alpha = 1.f;
@@ -209,55 +230,76 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 m_used = m_new;
             }
             const bool warp_rescale = __any_sync(0xffffffffu, need) && j > 0;
-            uint32_t pk[BN / 2];
-            float rs = 0.f;
-#pragma unroll
-            for (int i = 0; i < BN / 2; ++i) {
-                const float p0 = ex2_approx(fmaf(s[2 * i], sl2, -m_used));
-                const float p1 = ex2_approx(fmaf(s[2 * i + 1], sl2, -m_used));
-                pk[i] = pack_bf16(p0, p1);
-                rs += bf16lo(pk[i]) + bf16hi(pk[i]);
-            }
-            l += rs;
-            if (j >= 1) {   // P_{j-1} and O are in use by P V_{j-1} until it completes
-                ok = __all_sync(0xffffffffu, mbar_wait(&pv_done, (j - 1) & 1, abort_v, p.err));
+            if (j >= 1) {   // P_t and O_t are in use by P V_{t, j-1} until it completes
+                ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[t], (j - 1) & 1, abort_v, p.err));
                 if (!ok) break;
                 tc_fence_after();
             }
+            // pass 2: P = 2^(s*scale - m) per 64-key half (packed fp32 pairs),
+            // rounded to bf16 into the half's swizzled atom of the P buffer
+            const uint64_t scale2 = f2_pack(sl2, sl2);
+            const uint64_t negm2 = f2_pack(-m_used, -m_used);
+            uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-            for (int a = 0; a < 2; ++a)
+            for (int a = 0; a < 2; ++a) {
+                float sv[64];
+                tmem_ld32(tmem + lane_base + s_col + 64 * a, reinterpret_cast<uint32_t *>(sv));
+                tmem_ld32(tmem + lane_base + s_col + 64 * a + 32, reinterpret_cast<uint32_t *>(sv + 32));
+                tmem_ld_wait();
+                if (kvalid < 64 * (a + 1)) {
 #pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    const uint32_t *src = pk + a * 32 + c * 4;
-                    *reinterpret_cast<uint4 *>(prow + a * ATOM_BYTES + ((c ^ sw) << 4)) =
-                        make_uint4(src[0], src[1], src[2], src[3]);
+                    for (int i = 0; i < 64; ++i)
+                        if (64 * a + i >= kvalid) sv[i] = -INFINITY;
                 }
+                uint32_t pk[32];
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    float x0, x1;
+                    f2_unpack(f2_fma(f2_pack(sv[2 * i], sv[2 * i + 1]), scale2, negm2), x0, x1);
+                    const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+                    pk[i] = pack_bf16(p0, p1);
+                    acc2[i & 3] = f2_add(acc2[i & 3], f2_pack(p0, p1));
+                }
+#pragma unroll
+                for (int c = 0; c < 8; ++c)
+                    *reinterpret_cast<uint4 *>(prow + a * ATOM_BYTES + ((c ^ sw) << 4)) =
+                        make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+            }
+            {
+                float a0, a1;
+                f2_unpack(f2_add(f2_add(acc2[0], acc2[1]), f2_add(acc2[2], acc2[3])), a0, a1);
+                l += a0 + a1;
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s_free[t]);   // S_t may now be overwritten
             if (warp_rescale) {
 #pragma unroll
                 for (int c = 0; c < DH / 32; ++c) {
                     uint32_t o[32];
-                    tmem_ld32(tmem + lane_base + O_COL + 32 * c, o);
+                    tmem_ld32(tmem + lane_base + o_col + 32 * c, o);
                     tmem_ld_wait();
 #pragma unroll
                     for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-                    tmem_st32(tmem + lane_base + O_COL + 32 * c, o);
+                    tmem_st32(tmem + lane_base + o_col + 32 * c, o);
                 }
                 tmem_st_wait();
             }
             fence_proxy_async_smem();
             tc_fence_before();
-            mbar_arrive(&p_full);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&p_full[t]);
         }
-        if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&pv_done, (nb - 1) & 1, abort_v, p.err));
+        if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[t], (nb - 1) & 1, abort_v, p.err));
         if (ok) {
             tc_fence_after();
-            const int row = q0 + r;
+            const int row = q0 + t * BM + r;
             const float inv = 1.f / l;
             __nv_bfloat16 *dst = p.O + (int64_t)row * p.ldo + h * DH;
 #pragma unroll
             for (int c = 0; c < DH / 32; ++c) {
                 uint32_t o[32];
-                tmem_ld32(tmem + lane_base + O_COL + 32 * c, o);
+                tmem_ld32(tmem + lane_base + o_col + 32 * c, o);
                 tmem_ld_wait();
                 if (row < p.M) {
                     float f[32];
@@ -302,7 +344,7 @@ echo_status launch_dh(const void *Q, int64_t ldq, const void *K, const void *V, 
     p.O = static_cast<__nv_bfloat16 *>(O);
     p.ldo = ldo;
     p.err = echo::device_error_ptr();
-    dim3 grid((M + BM - 1) / BM, H);
+    dim3 grid((M + TILES * BM - 1) / (TILES * BM), H);
     echo::LaunchScope ls(ECHO_K_ATTENTION, M, L, (int64_t)H * DH, st);
     attn_tc_kernel<DH><<<grid, THREADS, Cfg<DH>::SMEM, st>>>(tq, tk, tv, p);
     return echo::last_launch_status();
