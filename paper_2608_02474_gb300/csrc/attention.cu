@@ -6,20 +6,22 @@
 // (two 128-query tiles, head), 12 warps, with the two tiles in ping-pong so
 // that one tile's softmax runs while the tensor cores work on the other:
 //   warp 0      TMA producer: both Q tiles once, then 128-key blocks K_0, V_0,
-//               K_1, V_1, ... (128-byte swizzle, 64-column boxes) into a
-//               three-slot ring shared by K and V;
+//               K_1, V_1, ... (128-byte swizzle, 64-column boxes) into a ring
+//               shared by K and V (5 slots for d = 128);
 //   warp 1      one thread issues S_t = Q_t K_j^T (M 128, N 128, K d) into the
-//               tile's TMEM S buffer and O_t += P_t V_j (M 128, N d, K 128; V is
-//               read MN-major straight from its row-major tile) into the tile's
-//               TMEM O accumulator, in the order PV0_j S0_{j+1} PV1_j S1_{j+1};
+//               tile's TMEM S columns and O_t += P_t V_j (M 128, N d, K 128; P
+//               read from TMEM, V read MN-major straight from its row-major
+//               tile) into the tile's TMEM O accumulator, in the order
+//               PV0_j S0_{j+1} PV1_j S1_{j+1};
 //   warp 2      allocates / frees 512 TMEM columns (S0, S1, O0, O1);
 //   warps 4..7  softmax of tile 0, warps 8..11 softmax of tile 1, one query row
-//               per thread (its TMEM lane): tcgen05.ld of the S row, online max,
-//               P = 2^(s*scale - m) rounded to bf16 into the tile's swizzled
-//               shared-memory P buffer (the A operand of P V), row sum of P; O is
-//               rescaled in TMEM only when the running max grows by more than
-//               2^8 (otherwise the stale max is kept, which is exact after the
-//               final division by the row sum); final O / l to bf16.
+//               per thread (its TMEM lane): pass 1 takes the row max of S, pass
+//               2 forms P = 2^(s*scale - m) on fp32 pairs, rounds it to bf16 and
+//               stores it back into the first 64 columns of S_t (over values it
+//               has already read); O is rescaled in TMEM only when the running
+//               max grows by more than 2^8 (otherwise the stale max is kept,
+//               which is exact after the final division by the row sum); final
+//               O / l to bf16.
 // Keys beyond L are masked to P = 0; queries beyond M run on zero rows and are
 // not stored.  Every mbarrier wait is bounded (ECHO_ERR_TIMEOUT).
 #include "common.cuh"
@@ -30,7 +32,7 @@ namespace {
 constexpr int BM = 128;        // queries per tile; two tiles per CTA
 constexpr int TILES = 2;
 constexpr int BN = 128;        // keys per block
-constexpr int RING = 3;        // K/V ring slots (K_j and V_j alternate)
+constexpr int RING_MAX = 8;    // K/V ring slots (K_j and V_j alternate)
 constexpr int THREADS = 384;   // 4 control warps + 2 softmax warpgroups
 constexpr uint32_t TMEM_COLS = 512;   // S0, S1, O0, O1
 constexpr uint32_t O_COL = 256;
@@ -42,8 +44,8 @@ struct Cfg {
     static constexpr int ATOMS = DH / 64;
     static constexpr int Q_BYTES = BM * DH * 2;
     static constexpr int SLOT_BYTES = BN * DH * 2;
-    static constexpr int P_BYTES = BM * BN * 2;
-    static constexpr int SMEM = TILES * Q_BYTES + RING * SLOT_BYTES + TILES * P_BYTES + 1024;
+    static constexpr int RING = DH == 128 ? 5 : RING_MAX;
+    static constexpr int SMEM = TILES * Q_BYTES + RING * SLOT_BYTES + 1024;
     static constexpr uint32_t IDESC_S = idesc_bf16_f32(BM, BN);
     static constexpr uint32_t IDESC_PV = idesc_bf16_f32(BM, DH) | (1u << 16);  // B MN-major
 };
@@ -64,14 +66,14 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                 ~static_cast<uintptr_t>(1023));
+    constexpr int RING = C::RING;
     uint8_t *Qs = smem;                                  // [TILES][Q_BYTES]
     uint8_t *Ring = Qs + TILES * C::Q_BYTES;             // [RING][SLOT_BYTES]
-    uint8_t *Ps = Ring + RING * C::SLOT_BYTES;           // [TILES][P_BYTES]
 
     // Every barrier is reused only after its previous phase has been observed
     // by its waiter, so no waiter can fall two phases behind.
-    __shared__ __align__(8) uint64_t q_full, ring_full[RING], ring_empty[RING];
-    __shared__ __align__(8) uint64_t s_full[TILES], s_free[TILES], p_full[TILES], pv_done[TILES];
+    __shared__ __align__(8) uint64_t q_full, ring_full[RING_MAX], ring_empty[RING_MAX];
+    __shared__ __align__(8) uint64_t s_full[TILES], p_full[TILES], pv_done[TILES];
     __shared__ __align__(8) uint64_t drain;
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_flag;
@@ -86,8 +88,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         for (int i = 0; i < RING; ++i) { mbar_init(&ring_full[i], 1); mbar_init(&ring_empty[i], 1); }
         for (int t = 0; t < TILES; ++t) {
             mbar_init(&s_full[t], 1);
-            mbar_init(&s_free[t], 4);    // one arrival per softmax warp
-            mbar_init(&p_full[t], 4);
+            mbar_init(&p_full[t], 4);    // one arrival per softmax warp
             mbar_init(&pv_done[t], 1);
         }
         mbar_init(&drain, 1);
@@ -131,10 +132,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer ----------------
         // order: S0_0 S1_0 | PV0_0 S0_1 PV1_0 S1_1 | PV0_1 S0_2 PV1_1 S1_2 | ...
+        // P_t lives in the first 64 columns of S_t; S_t of the next block is
+        // issued after P V of this block, and tcgen05.mma from one thread run in
+        // order, so the S write cannot overtake the P read.  The commit of S_t
+        // (s_full) therefore also tells the softmax that P V_{t, j-1} is done.
         bool ok = mbar_wait(&q_full, 0, abort_v, p.err);
         auto issue_s = [&](int t, int j) -> bool {
             const int li = 2 * j, slot = li % RING;
-            if (j > 0 && !mbar_wait(&s_free[t], (j - 1) & 1, abort_v, p.err)) return false;
             if (!mbar_wait(&ring_full[slot], (li / RING) & 1, abort_v, p.err)) return false;
             tc_fence_after();
             const uint8_t *qt = Qs + t * C::Q_BYTES;
@@ -154,16 +158,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             if (!mbar_wait(&p_full[t], j & 1, abort_v, p.err)) return false;
             if (!mbar_wait(&ring_full[slot], (li / RING) & 1, abort_v, p.err)) return false;
             tc_fence_after();
-            const uint8_t *pt = Ps + t * C::P_BYTES;
             const uint8_t *vt = Ring + slot * C::SLOT_BYTES;
 #pragma unroll
-            for (int kk = 0; kk < BN / 16; ++kk) {
-                const int a = kk >> 2, off = (kk & 3) * 32;
-                tc_mma_f16(tmem + O_COL + (uint32_t)(t * DH), smem_desc_sw128(pt + a * ATOM_BYTES + off),
-                           smem_desc_sw128_mn(vt + kk * 2048, ATOM_BYTES, 1024), C::IDESC_PV,
-                           (j > 0 || kk > 0) ? 1u : 0u);
-            }
-            tc_commit(&pv_done[t]);
+            for (int kk = 0; kk < BN / 16; ++kk)
+                tc_mma_f16_tmem_a(tmem + O_COL + (uint32_t)(t * DH), tmem + (uint32_t)(t * BN + 8 * kk),
+                                  smem_desc_sw128_mn(vt + kk * 2048, ATOM_BYTES, 1024), C::IDESC_PV,
+                                  (j > 0 || kk > 0) ? 1u : 0u);
+            if (j == nb - 1) tc_commit(&pv_done[t]);            // O_t is final
             if (t == TILES - 1) tc_commit(&ring_empty[slot]);   // V_j no longer needed
             return true;
         };
@@ -189,8 +190,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         const float sl2 = p.scale_log2;
         float m_used = -INFINITY, l = 0.f;
         bool ok = true;
-        uint8_t *prow = Ps + t * C::P_BYTES + r * 128;
-        const int sw = r & 7;
         for (int j = 0; j < nb; ++j) {
             ok = __all_sync(0xffffffffu, mbar_wait(&s_full[t], j & 1, abort_v, p.err));
             if (!ok) break;
@@ -230,49 +229,40 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 m_used = m_new;
             }
             const bool warp_rescale = __any_sync(0xffffffffu, need) && j > 0;
-            if (j >= 1) {   // P_t and O_t are in use by P V_{t, j-1} until it completes
-                ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[t], (j - 1) & 1, abort_v, p.err));
-                if (!ok) break;
-                tc_fence_after();
-            }
-            // pass 2: P = 2^(s*scale - m) per 64-key half (packed fp32 pairs),
-            // rounded to bf16 into the half's swizzled atom of the P buffer
+            // (S_t of this block completed after P V_{t, j-1}: O_t is settled and
+            // the P columns are free)
+            // pass 2: P = 2^(s*scale - m) per 32-key chunk (packed fp32 pairs),
+            // rounded to bf16 pairs into TMEM columns [16 c, 16 c + 16) of S_t,
+            // i.e. over S values this pass has already read
             const uint64_t scale2 = f2_pack(sl2, sl2);
             const uint64_t negm2 = f2_pack(-m_used, -m_used);
             uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-            for (int a = 0; a < 2; ++a) {
-                float sv[64];
-                tmem_ld32(tmem + lane_base + s_col + 64 * a, reinterpret_cast<uint32_t *>(sv));
-                tmem_ld32(tmem + lane_base + s_col + 64 * a + 32, reinterpret_cast<uint32_t *>(sv + 32));
+            for (int c = 0; c < BN / 32; ++c) {
+                float sv[32];
+                tmem_ld32(tmem + lane_base + s_col + 32 * c, reinterpret_cast<uint32_t *>(sv));
                 tmem_ld_wait();
-                if (kvalid < 64 * (a + 1)) {
+                if (kvalid < 32 * (c + 1)) {
 #pragma unroll
-                    for (int i = 0; i < 64; ++i)
-                        if (64 * a + i >= kvalid) sv[i] = -INFINITY;
+                    for (int i = 0; i < 32; ++i)
+                        if (32 * c + i >= kvalid) sv[i] = -INFINITY;
                 }
-                uint32_t pk[32];
+                uint32_t pk[16];
 #pragma unroll
-                for (int i = 0; i < 32; ++i) {
+                for (int i = 0; i < 16; ++i) {
                     float x0, x1;
                     f2_unpack(f2_fma(f2_pack(sv[2 * i], sv[2 * i + 1]), scale2, negm2), x0, x1);
                     const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
                     pk[i] = pack_bf16(p0, p1);
                     acc2[i & 3] = f2_add(acc2[i & 3], f2_pack(p0, p1));
                 }
-#pragma unroll
-                for (int c = 0; c < 8; ++c)
-                    *reinterpret_cast<uint4 *>(prow + a * ATOM_BYTES + ((c ^ sw) << 4)) =
-                        make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+                tmem_st16(tmem + lane_base + s_col + 16 * c, pk);
             }
             {
                 float a0, a1;
                 f2_unpack(f2_add(f2_add(acc2[0], acc2[1]), f2_add(acc2[2], acc2[3])), a0, a1);
                 l += a0 + a1;
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&s_free[t]);   // S_t may now be overwritten
             if (warp_rescale) {
 #pragma unroll
                 for (int c = 0; c < DH / 32; ++c) {
@@ -285,12 +275,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 }
                 tmem_st_wait();
             }
-            fence_proxy_async_smem();
+            tmem_st_wait();
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&p_full[t]);
         }
-        if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[t], (nb - 1) & 1, abort_v, p.err));
+        if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[t], 0, abort_v, p.err));
         if (ok) {
             tc_fence_after();
             const int row = q0 + t * BM + r;
