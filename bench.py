@@ -44,6 +44,9 @@ def parse():
     ap.add_argument("--profile", default="audio", help="audio profile")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="refresh-ratio x audio-profile sweep against the uncached block "
+                         "(one JSON line per point and a break-even summary)")
     return ap.parse_args()
 
 
@@ -131,11 +134,10 @@ def roofline(records, K, peaks):
         b[0] += cnt
         b[1] += ms
     total = sum(v[1] for v in by_kernel.values())
-    dom = max(by_kernel, key=lambda x: by_kernel[x][1])
-    # the dominant kernel's largest launch shape (most time)
-    shapes = [(ms / cnt, cnt, key) for key, (cnt, ms) in agg.items() if key[0] == dom]
-    shape = max(shapes, key=lambda s: s[0] * s[1])
-    avg_ms, cnt, (name, m, n, k) = shape
+    # the dominant kernel: the (kernel, launch shape) with the largest share of the step
+    key = max(agg, key=lambda kk: agg[kk][1])
+    cnt, tot_ms = agg[key]
+    avg_ms, (name, m, n, k) = tot_ms / cnt, key
     flops, byts = algorithmic_work(name, m, n, k, K)
     traffic = measured_traffic(name, [m, n, k])
     if flops is not None:
@@ -285,6 +287,72 @@ def run_reference(args, w, rnum, rden, rank):
     print(json.dumps(line), flush=True)
 
 
+def run_sweep(args, w, blocks, x0, xs, dev, rank, world):
+    """Cached step time for every (audio profile, ratio) and the uncached block."""
+    import torch
+    from paper_2608_02474_gb300 import echocache as ec
+    from paper_2608_02474_gb300.pipeline import CachedStack
+    from synth import generate as G
+
+    profiles = w.sweep_profiles or (args.profile,)
+    ratios = w.sweep_ratios or ((w.ratio_num, w.ratio_den),)
+    stack = CachedStack(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc, blocks, device=dev)
+    x0_d = torch.from_numpy(x0).to(dev, torch.bfloat16)
+    xs_d = [torch.from_numpy(x).to(dev, torch.bfloat16) for x in xs]
+    stream = torch.cuda.current_stream()
+
+    def timed(fn, steps):
+        for i in range(args.warmup):
+            fn(i)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(steps):
+            fn(i)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        assert ec.echo_get_device_error() == 0
+        return e0.elapsed_time(e1) / steps
+
+    summary = {}
+    for prof in profiles:
+        audio_d = torch.from_numpy(G.audio(w, prof)).to(dev)
+        stack.set_audio(audio_d)
+        # uncached comparator: every token refreshed (K = NT), same kernels
+        full_ms = timed(lambda i: stack.step(xs_d[i % 2], 1, 1, full=True), args.steps)
+        stack.step(x0_d, 1, 1, full=True)
+        points = []
+        for num, den in ratios:
+            def one(i, num=num, den=den):
+                stack.set_audio(audio_d)
+                return stack.step(xs_d[i % 2], num, den)
+            ms = timed(one, args.steps)
+            K = (num * w.NT + den - 1) // den
+            points.append((num / den, ms))
+            if rank == 0:
+                print(json.dumps({"sweep": w.name, "profile": prof, "ratio": f"{num}/{den}",
+                                  "active_tokens": K, "ms_per_step": round(ms, 4),
+                                  "tokens_per_s": round(world * w.NT / (ms * 1e-3), 1),
+                                  "uncached_ms": round(full_ms, 4),
+                                  "speedup_vs_uncached": round(full_ms / ms, 3)}), flush=True)
+        # smallest ratio where the cached step is no faster than the uncached one
+        be = None
+        for (r0, m0), (r1, m1) in zip(points, points[1:]):
+            if m0 < full_ms <= m1:
+                be = r0 + (r1 - r0) * (full_ms - m0) / (m1 - m0)
+                break
+        if be is None and points and points[0][1] >= full_ms:
+            be = points[0][0]
+        summary[prof] = {"uncached_ms": round(full_ms, 4),
+                         "break_even_ratio": None if be is None else round(be, 4)}
+    if rank == 0:
+        print(json.dumps({"sweep_summary": w.name, "tokens": w.NT, "profiles": summary,
+                          "note": "break_even_ratio = smallest refresh ratio at which the cached "
+                                  "step is no faster than the uncached block (linear "
+                                  "interpolation); null = cached faster at every ratio tried"}),
+              flush=True)
+
+
 def main():
     args = parse()
     from synth import ALL
@@ -317,7 +385,12 @@ def main():
             dist.barrier()
 
     audio, W, cond, x0, xs = build_inputs(w, args.profile)
-    blocks = [ec.DeviceBlock.from_host(W, cond, device=dev) for _ in range(w.layers)]
+    from synth import generate as G
+    blocks = [ec.DeviceBlock.from_host(W if l == 0 else G.block_weights(w, l), cond, device=dev)
+              for l in range(w.layers)]
+    if args.sweep:
+        run_sweep(args, w, blocks, x0, xs, dev, rank, world)
+        return
     stack = CachedStack(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc, blocks, device=dev)
     audio_d = torch.from_numpy(audio).to(dev)
     x0_d = torch.from_numpy(x0).to(dev, torch.bfloat16)
@@ -371,21 +444,20 @@ def main():
     roof, table = roofline(records, K, peaks)
 
     # ---- end to end through the public API with host buffers ----
+    # every step uploads its input from pinned host memory and downloads its
+    # output into pinned host memory (CachedStack.run_host overlaps those
+    # copies with the neighbouring steps' compute)
     e2e = None
     if not args.no_e2e:
         xh = [torch.from_numpy(x).to(torch.bfloat16).pin_memory() for x in xs]
-        yh = torch.empty(w.NT, w.D, dtype=torch.bfloat16).pin_memory()
-        xd = torch.empty(w.NT, w.D, dtype=torch.bfloat16, device=dev)
-        for i in range(2):
-            xd.copy_(xh[i % 2], non_blocking=True)
-            yh.copy_(one_step(xd), non_blocking=True)
+        yh = [torch.empty(w.NT, w.D, dtype=torch.bfloat16).pin_memory() for _ in range(2)]
+        stack.run_host([xh[0], xh[1]], yh, rnum, rden, audio=audio_d)
         torch.cuda.synchronize()
         barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        for i in range(args.steps):
-            xd.copy_(xh[i % 2], non_blocking=True)
-            yh.copy_(one_step(xd), non_blocking=True)
+        stack.run_host([xh[i % 2] for i in range(args.steps)],
+                       [yh[i % 2] for i in range(args.steps)], rnum, rden, audio=audio_d)
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
@@ -395,7 +467,7 @@ def main():
             dist.all_reduce(t, op=dist.ReduceOp.MAX)
             ems = float(t.item())
         e2e = {"value": round(world * w.NT / (ems * 1e-3), 2), "unit": UNIT,
-               "h2d_bytes_per_step": xh[0].numel() * 2, "d2h_bytes_per_step": yh.numel() * 2,
+               "h2d_bytes_per_step": xh[0].numel() * 2, "d2h_bytes_per_step": yh[0].numel() * 2,
                "ms_per_step": round(ems, 3)}
 
     cpu = None

@@ -45,10 +45,12 @@ class CachedStack:
         return self.band, self.seg
 
     def step(self, x: torch.Tensor, ratio_num: int, ratio_den: int, full: bool = False,
-             keep_scores: bool = False) -> torch.Tensor:
-        """One denoising step over every layer; returns the last layer's output."""
+             keep_scores: bool = False, out: torch.Tensor | None = None) -> torch.Tensor:
+        """One denoising step over every layer; returns the last layer's output
+        (written into `out` when given)."""
         cur = x
         self.last_K = []
+        last = len(self.blocks) - 1
         for l, blk in enumerate(self.blocks):
             if full:
                 idx, K = self.all_idx, self.NT
@@ -58,9 +60,53 @@ class CachedStack:
                                            self.mode, idx=self.idx,
                                            scores=self.scores if keep_scores else None,
                                            workspace=self.sel_ws)
-            out = self.y[l % 2]
+            dst = out if (l == last and out is not None) else self.y[l % 2]
             ec.echo_block_step(blk, self.dims, cur, idx, K, self.cache_q[l], self.cache_s[l],
-                               y=out, workspace=self.ws)
+                               y=dst, workspace=self.ws)
             self.last_K.append(K)
-            cur = out
+            cur = dst
         return cur
+
+    def run_host(self, host_x: list, host_y: list, ratio_num: int, ratio_den: int,
+                 audio: torch.Tensor | None = None):
+        """Steps whose inputs and outputs live in pinned host memory.
+
+        Step i copies host_x[i] to the device, runs one step (the audio energy
+        first when `audio` is given) and copies the result into host_y[i].  The
+        copies run on their own streams into double-buffered device tensors, so
+        the upload of step i+1 and the download of step i-1 overlap step i.
+        Returns after everything has been enqueued; synchronise before reading
+        host_y."""
+        dev = self.seg.device
+        comp = torch.cuda.current_stream(dev)
+        if not hasattr(self, "_h2d"):
+            self._h2d, self._d2h = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+            self._xd = [torch.empty(self.NT, self.D, dtype=torch.bfloat16, device=dev) for _ in range(2)]
+            self._yd = [torch.empty(self.NT, self.D, dtype=torch.bfloat16, device=dev) for _ in range(2)]
+            self._ev = {k: [torch.cuda.Event() for _ in range(2)]
+                        for k in ("x_ready", "x_used", "y_ready", "y_copied")}
+            for k in ("x_used", "y_copied"):
+                for e in self._ev[k]:
+                    e.record(comp)
+        ev = self._ev
+        start = torch.cuda.Event()
+        start.record(comp)                  # copies start after work already queued
+        self._h2d.wait_event(start)
+        for i, (hx, hy) in enumerate(zip(host_x, host_y)):
+            b = i % 2
+            with torch.cuda.stream(self._h2d):
+                self._h2d.wait_event(ev["x_used"][b])
+                self._xd[b].copy_(hx, non_blocking=True)
+                ev["x_ready"][b].record(self._h2d)
+            comp.wait_event(ev["x_ready"][b])
+            comp.wait_event(ev["y_copied"][b])
+            if audio is not None:
+                self.set_audio(audio)
+            self.step(self._xd[b], ratio_num, ratio_den, out=self._yd[b])
+            ev["x_used"][b].record(comp)
+            ev["y_ready"][b].record(comp)
+            with torch.cuda.stream(self._d2h):
+                self._d2h.wait_event(ev["y_ready"][b])
+                hy.copy_(self._yd[b], non_blocking=True)
+                ev["y_copied"][b].record(self._d2h)
+        comp.wait_event(ev["y_copied"][(len(host_x) - 1) % 2])

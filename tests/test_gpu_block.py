@@ -181,3 +181,34 @@ def test_wan_block_sampled_rows(ec):
     res = R()
     res.idx, res.y_act_rows = oidx, ya
     check_layer(ec, w, res, q, s, g_idx, y, qd, sd, rows=rows)
+
+
+def test_pipeline_host_buffers_match_device_steps(ec):
+    """CachedStack.run_host (pinned host in/out, copies overlapped with compute)
+    returns exactly what the same steps return from device tensors."""
+    from paper_2608_02474_gb300.pipeline import CachedStack
+    w = TINY_256
+    audio = G.audio(w)
+    W = G.block_weights(w, 0)
+    cond = G.cond_tokens(w, audio)
+    x0 = G.latents(w)
+    xs = [G.step_input(w, x0, t) for t in (1, 2, 3)]
+    blk = ec.DeviceBlock.from_host(W, cond)
+    ad = torch.from_numpy(audio).to(DEV)
+    outs = []
+    for mode in ("device", "host"):
+        st = CachedStack(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc, [blk], device=DEV)
+        st.set_audio(ad)
+        st.step(bf(x0), 1, 1, full=True)
+        if mode == "device":
+            outs.append([st.step(bf(x), w.ratio_num, w.ratio_den).float().cpu().numpy().copy()
+                         for x in xs])
+        else:
+            hx = [torch.from_numpy(x).to(torch.bfloat16).pin_memory() for x in xs]
+            hy = [torch.empty(w.NT, w.D, dtype=torch.bfloat16).pin_memory() for _ in xs]
+            st.run_host(hx, hy, w.ratio_num, w.ratio_den)
+            torch.cuda.synchronize()
+            outs.append([y.float().numpy().copy() for y in hy])
+    for a, b in zip(*outs):
+        assert np.array_equal(a, b)
+    assert ec.echo_get_device_error() == 0
