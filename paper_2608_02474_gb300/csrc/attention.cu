@@ -15,10 +15,10 @@
 //               PV0_j S0_{j+1} PV1_j S1_{j+1};
 //   warp 2      allocates / frees 512 TMEM columns (S0, S1, O0, O1);
 //   warps 4..7  softmax of tile 0, warps 8..11 softmax of tile 1, one query row
-//               per thread (its TMEM lane): pass 1 takes the row max of S, pass
-//               2 forms P = 2^(s*scale - m) on fp32 pairs, rounds it to bf16 and
-//               stores it back into the first 64 columns of S_t (over values it
-//               has already read); O is rescaled in TMEM only when the running
+//               per thread (its TMEM lane, 224 registers after setmaxnreg): the
+//               S row is loaded once, its max taken, P = 2^(s*scale - m) formed
+//               on fp32 pairs, rounded to bf16 and stored back into the first 64
+//               columns of S_t; O is rescaled in TMEM only when the running
 //               max grows by more than 2^8 (otherwise the stale max is kept,
 //               which is exact after the final division by the row sum); final
 //               O / l to bf16.
@@ -104,7 +104,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
     volatile int *abort_v = &abort_flag;
-
+    // Register split (launch: 384 x 168 = 64512): the control warpgroup keeps
+    // 48 per thread, the two softmax warpgroups take 224 (128*48 + 256*224 = 63488).
+    if (warp < 4) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 48;" ::: "memory");
     if (warp == 0 && lane == 0) {
         // ---------------- TMA producer: Q0, Q1, then K_0, V_0, K_1, V_1, ... ----------------
         const int x0 = h * DH;
@@ -179,7 +182,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             tc_commit(&drain);
             mbar_wait(&drain, 0, abort_v, nullptr, 100000000ull);
         }
-    } else if (warp >= 4) {
+    }
+    } else {
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 224;" ::: "memory");
         // ---------------- softmax / correction / epilogue of tile t ----------------
         const int t = (warp - 4) >> 2;
         const int quad = warp & 3;
@@ -194,32 +199,27 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             ok = __all_sync(0xffffffffu, mbar_wait(&s_full[t], j & 1, abort_v, p.err));
             if (!ok) break;
             tc_fence_after();
-            // pass 1: row max over the 128 keys of the block (3-input max)
+            // the whole S row of this block in registers (one TMEM round trip)
             const int kvalid = p.L - j * BN;                 // keys of this block that exist
-            float mx;
-            {
-                float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+            float sv[BN];
 #pragma unroll
-                for (int c = 0; c < BN / 64; ++c) {
-                    float sv[64];
-                    tmem_ld32(tmem + lane_base + s_col + 64 * c, reinterpret_cast<uint32_t *>(sv));
-                    tmem_ld32(tmem + lane_base + s_col + 64 * c + 32, reinterpret_cast<uint32_t *>(sv + 32));
-                    tmem_ld_wait();
-                    if (kvalid < 64 * (c + 1)) {                 // tail block only
+            for (int c = 0; c < BN / 32; ++c)
+                tmem_ld32(tmem + lane_base + s_col + 32 * c, reinterpret_cast<uint32_t *>(sv + 32 * c));
+            tmem_ld_wait();
+            if (kvalid < BN) {                               // tail block only
 #pragma unroll
-                        for (int i = 0; i < 64; ++i)
-                            if (64 * c + i >= kvalid) sv[i] = -INFINITY;
-                    }
-#pragma unroll
-                    for (int i = 0; i < 64; i += 8) {
-                        m4[0] = fmax3(m4[0], sv[i], sv[i + 1]);
-                        m4[1] = fmax3(m4[1], sv[i + 2], sv[i + 3]);
-                        m4[2] = fmax3(m4[2], sv[i + 4], sv[i + 5]);
-                        m4[3] = fmax3(m4[3], sv[i + 6], sv[i + 7]);
-                    }
-                }
-                mx = fmaxf(fmax3(m4[0], m4[1], m4[2]), m4[3]);
+                for (int i = 0; i < BN; ++i)
+                    if (i >= kvalid) sv[i] = -INFINITY;
             }
+            float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+            for (int i = 0; i < BN; i += 8) {
+                m4[0] = fmax3(m4[0], sv[i], sv[i + 1]);
+                m4[1] = fmax3(m4[1], sv[i + 2], sv[i + 3]);
+                m4[2] = fmax3(m4[2], sv[i + 4], sv[i + 5]);
+                m4[3] = fmax3(m4[3], sv[i + 6], sv[i + 7]);
+            }
+            const float mx = fmaxf(fmax3(m4[0], m4[1], m4[2]), m4[3]);
             const float m_new = fmaxf(m_used, mx * sl2);
             const bool need = m_new > m_used + RESCALE_LOG2;
             float alpha = 1.f;
@@ -231,33 +231,22 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             const bool warp_rescale = __any_sync(0xffffffffu, need) && j > 0;
             // (S_t of this block completed after P V_{t, j-1}: O_t is settled and
             // the P columns are free)
-            // pass 2: P = 2^(s*scale - m) per 32-key chunk (packed fp32 pairs),
-            // rounded to bf16 pairs into TMEM columns [16 c, 16 c + 16) of S_t,
-            // i.e. over S values this pass has already read
+            // P = 2^(s*scale - m) on fp32 pairs, rounded to bf16 pairs and stored
+            // into TMEM columns [0, 64) of S_t (S is already in registers)
             const uint64_t scale2 = f2_pack(sl2, sl2);
             const uint64_t negm2 = f2_pack(-m_used, -m_used);
             uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
+            uint32_t pk[BN / 2];
 #pragma unroll
-            for (int c = 0; c < BN / 32; ++c) {
-                float sv[32];
-                tmem_ld32(tmem + lane_base + s_col + 32 * c, reinterpret_cast<uint32_t *>(sv));
-                tmem_ld_wait();
-                if (kvalid < 32 * (c + 1)) {
-#pragma unroll
-                    for (int i = 0; i < 32; ++i)
-                        if (32 * c + i >= kvalid) sv[i] = -INFINITY;
-                }
-                uint32_t pk[16];
-#pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    float x0, x1;
-                    f2_unpack(f2_fma(f2_pack(sv[2 * i], sv[2 * i + 1]), scale2, negm2), x0, x1);
-                    const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
-                    pk[i] = pack_bf16(p0, p1);
-                    acc2[i & 3] = f2_add(acc2[i & 3], f2_pack(p0, p1));
-                }
-                tmem_st16(tmem + lane_base + s_col + 16 * c, pk);
+            for (int i = 0; i < BN / 2; ++i) {
+                float x0, x1;
+                f2_unpack(f2_fma(f2_pack(sv[2 * i], sv[2 * i + 1]), scale2, negm2), x0, x1);
+                const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+                pk[i] = pack_bf16(p0, p1);
+                acc2[i & 3] = f2_add(acc2[i & 3], f2_pack(p0, p1));
             }
+            tmem_st32(tmem + lane_base + s_col, pk);
+            tmem_st32(tmem + lane_base + s_col + 32, pk + 32);
             {
                 float a0, a1;
                 f2_unpack(f2_add(f2_add(acc2[0], acc2[1]), f2_add(acc2[2], acc2[3])), a0, a1);
