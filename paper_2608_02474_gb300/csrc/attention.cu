@@ -18,10 +18,10 @@
 //               per thread (its TMEM lane, 224 registers after setmaxnreg): the
 //               S row is loaded once, its max taken, P = 2^(s*scale - m) formed
 //               on fp32 pairs, rounded to bf16 and stored back into the first 64
-//               columns of S_t; O is rescaled in TMEM only when the running
-//               max grows by more than 2^8 (otherwise the stale max is kept,
-//               which is exact after the final division by the row sum); final
-//               O / l to bf16.
+//               columns of S_t.  The running max comes from the first block;
+//               later blocks reuse it (exact after the final division by the row
+//               sum) and redo themselves with a fresh max, rescaling O in TMEM,
+//               only when their row sum shows P above 2^64; final O / l to bf16.
 // Keys beyond L are masked to P = 0; queries beyond M run on zero rows and are
 // not stored.  Every mbarrier wait is bounded (ECHO_ERR_TIMEOUT).
 #include "common.cuh"
@@ -37,7 +37,6 @@ constexpr int THREADS = 384;   // 4 control warps + 2 softmax warpgroups
 constexpr uint32_t TMEM_COLS = 512;   // S0, S1, O0, O1
 constexpr uint32_t O_COL = 256;
 constexpr int ATOM_BYTES = 128 * 128;   // one [128 rows x 64 bf16] 128B-swizzled box
-constexpr float RESCALE_LOG2 = 8.f;
 
 template <int DH>
 struct Cfg {
@@ -211,59 +210,72 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 for (int i = 0; i < BN; ++i)
                     if (i >= kvalid) sv[i] = -INFINITY;
             }
-            float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+            // The running max m_used is taken from the first block only.  Later
+            // blocks form P with it directly: the result is exact after the final
+            // division by the row sum, and fp32 / bf16 keep their precision at any
+            // exponent, so a rescale is needed only when P could overflow.  The
+            // block's row sum bounds its largest P; when it exceeds 2^64 (or is
+            // not finite) the block is redone with a fresh max and O, l rescaled.
+            auto block_max = [&]() -> float {
+                float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-            for (int i = 0; i < BN; i += 8) {
-                m4[0] = fmax3(m4[0], sv[i], sv[i + 1]);
-                m4[1] = fmax3(m4[1], sv[i + 2], sv[i + 3]);
-                m4[2] = fmax3(m4[2], sv[i + 4], sv[i + 5]);
-                m4[3] = fmax3(m4[3], sv[i + 6], sv[i + 7]);
-            }
-            const float mx = fmaxf(fmax3(m4[0], m4[1], m4[2]), m4[3]);
-            const float m_new = fmaxf(m_used, mx * sl2);
-            const bool need = m_new > m_used + RESCALE_LOG2;
-            float alpha = 1.f;
-            if (need) {
-                alpha = ex2_approx(m_used - m_new);
-                l *= alpha;
-                m_used = m_new;
-            }
-            const bool warp_rescale = __any_sync(0xffffffffu, need) && j > 0;
-            // (S_t of this block completed after P V_{t, j-1}: O_t is settled and
-            // the P columns are free)
-            // P = 2^(s*scale - m) on fp32 pairs, rounded to bf16 pairs and stored
-            // into TMEM columns [0, 64) of S_t (S is already in registers)
-            const uint64_t scale2 = f2_pack(sl2, sl2);
-            const uint64_t negm2 = f2_pack(-m_used, -m_used);
-            uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
+                for (int i = 0; i < BN; i += 8) {
+                    m4[0] = fmax3(m4[0], sv[i], sv[i + 1]);
+                    m4[1] = fmax3(m4[1], sv[i + 2], sv[i + 3]);
+                    m4[2] = fmax3(m4[2], sv[i + 4], sv[i + 5]);
+                    m4[3] = fmax3(m4[3], sv[i + 6], sv[i + 7]);
+                }
+                return fmaxf(fmax3(m4[0], m4[1], m4[2]), m4[3]);
+            };
+            // P = 2^(s*scale - m) on fp32 pairs, rounded to bf16 pairs; returns
+            // the row sum of this block
             uint32_t pk[BN / 2];
+            auto exp_pass = [&]() -> float {
+                const uint64_t scale2 = f2_pack(sl2, sl2);
+                const uint64_t negm2 = f2_pack(-m_used, -m_used);
+                uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-            for (int i = 0; i < BN / 2; ++i) {
-                float x0, x1;
-                f2_unpack(f2_fma(f2_pack(sv[2 * i], sv[2 * i + 1]), scale2, negm2), x0, x1);
-                const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
-                pk[i] = pack_bf16(p0, p1);
-                acc2[i & 3] = f2_add(acc2[i & 3], f2_pack(p0, p1));
-            }
-            tmem_st32(tmem + lane_base + s_col, pk);
-            tmem_st32(tmem + lane_base + s_col + 32, pk + 32);
-            {
+                for (int i = 0; i < BN / 2; ++i) {
+                    float x0, x1;
+                    f2_unpack(f2_fma(f2_pack(sv[2 * i], sv[2 * i + 1]), scale2, negm2), x0, x1);
+                    const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+                    pk[i] = pack_bf16(p0, p1);
+                    acc2[i & 3] = f2_add(acc2[i & 3], f2_pack(p0, p1));
+                }
                 float a0, a1;
                 f2_unpack(f2_add(f2_add(acc2[0], acc2[1]), f2_add(acc2[2], acc2[3])), a0, a1);
-                l += a0 + a1;
-            }
-            if (warp_rescale) {
-#pragma unroll
-                for (int c = 0; c < DH / 32; ++c) {
-                    uint32_t o[32];
-                    tmem_ld32(tmem + lane_base + o_col + 32 * c, o);
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-                    tmem_st32(tmem + lane_base + o_col + 32 * c, o);
+                return a0 + a1;
+            };
+            if (j == 0) m_used = block_max() * sl2;
+            float bsum = exp_pass();
+            const bool redo = !(bsum <= 1.8446744e19f);     // > 2^64, inf or NaN
+            if (__any_sync(0xffffffffu, redo)) {              // rare: warp-uniform slow path
+                float alpha = 1.f;
+                if (redo) {
+                    const float m_new = fmaxf(m_used, block_max() * sl2);
+                    alpha = ex2_approx(m_used - m_new);
+                    l *= alpha;
+                    m_used = m_new;
                 }
-                tmem_st_wait();
+                if (j > 0) {   // S_t of this block completed after P V_{t, j-1}: O_t is settled
+#pragma unroll
+                    for (int c = 0; c < DH / 32; ++c) {
+                        uint32_t o[32];
+                        tmem_ld32(tmem + lane_base + o_col + 32 * c, o);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+                        tmem_st32(tmem + lane_base + o_col + 32 * c, o);
+                    }
+                    tmem_st_wait();
+                }
+                bsum = exp_pass();
             }
+            l += bsum;
+            // P into TMEM columns [0, 64) of S_t (S is already in registers)
+            tmem_st32(tmem + lane_base + s_col, pk);
+            tmem_st32(tmem + lane_base + s_col + 32, pk + 32);
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();

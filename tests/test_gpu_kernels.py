@@ -284,3 +284,24 @@ def test_attention(ec, M, L, H, d):
                            KV[:, D:].astype(np.float64), H)
     close_bf16(out.float().cpu().numpy(), ref)
     no_device_error(ec)
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_attention_running_max_jumps(ec, d):
+    """Later key blocks whose logits exceed the first block's by far more than
+    2^64 force the kernel's rescale path (running max refreshed, O and the row
+    sum rescaled in tensor memory); the result must still match the oracle."""
+    H, M, L = 2, 150, 700
+    D = H * d
+    g = np.random.default_rng(d)
+    Q = np.full((M, D), 2.0, dtype=F32) + g.standard_normal((M, D)).astype(F32) * F32(0.05)
+    K = g.standard_normal((L, D)).astype(F32) * F32(0.1)
+    K[400:] += F32(3.0)                          # logits jump by ~ 6 d / sqrt(d) nats
+    V = g.standard_normal((L, D)).astype(F32)
+    Q, K, V = (G.to_bf16_values(a) for a in (Q, K, V))
+    KV = np.concatenate([K, V], axis=1)
+    kvd = bf(KV)
+    out = ec.echo_attention(bf(Q), kvd[:, :D], kvd[:, D:], H, d)
+    ref = oracle.block.mha(Q.astype(np.float64), K.astype(np.float64), V.astype(np.float64), H)
+    close_bf16(out.float().cpu().numpy(), ref)
+    no_device_error(ec)
