@@ -2,9 +2,11 @@
 // an optional row gather: out[j] = LN(in[rows[j]]).  The gathered form is the
 // "select active latents" step of Sec. 3.3 fused with the LN that follows it.
 //
-// A row lives in registers (up to 8 chunks of 8 values per thread): one warp
-// per row for D <= 1024, four warps per row up to D = 8192.  Mean first, then
-// the centred variance, both fp32 tree reductions; one HBM read, one write.
+// A row lives in registers: for bf16 input one warp per row holds it packed (up
+// to 32 16-byte chunks per lane); for fp32 input up to 8 chunks of 8 values per
+// thread, one warp per row for D <= 1024, four warps per row up to D = 8192.
+// Mean first, then the centred variance, both fp32 tree reductions; one HBM
+// read, one write.
 #include "common.cuh"
 #include "internal.h"
 
@@ -103,11 +105,91 @@ layernorm_kernel(const T *__restrict__ in, const int32_t *__restrict__ rows, int
     }
 }
 
+// bf16 input: one warp per row, the row held packed in registers (CPL 16-byte
+// chunks per lane), so each row is read from HBM once and no block barrier is
+// needed.
+template <int CPL>
+__global__ void __launch_bounds__(kThreads)
+layernorm_warp_bf16(const __nv_bfloat16 *__restrict__ in, const int32_t *__restrict__ rows,
+                    int n_rows, int D, __nv_bfloat16 *__restrict__ out) {
+    const int lane = threadIdx.x & 31;
+    const int warps = kThreads / 32;
+    const int C = D >> 3;
+    const float invD = 1.f / (float)D;
+    for (int j = blockIdx.x * warps + (threadIdx.x >> 5); j < n_rows; j += gridDim.x * warps) {
+        const int r = rows ? rows[j] : j;
+        const uint4 *src = reinterpret_cast<const uint4 *>(in + (int64_t)r * D);
+        uint4 v[CPL];
+#pragma unroll
+        for (int k = 0; k < CPL; ++k) {
+            const int c = lane + 32 * k;
+            v[k] = c < C ? __ldcs(src + c) : make_uint4(0, 0, 0, 0);
+        }
+        float s = 0.f;
+#pragma unroll
+        for (int k = 0; k < CPL; ++k) {
+            float f[8];
+            unpack8_bf16(v[k], f);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) s += f[e];
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        const float mean = s * invD;
+        float ss = 0.f;
+#pragma unroll
+        for (int k = 0; k < CPL; ++k) {
+            if (lane + 32 * k < C) {
+                float f[8];
+                unpack8_bf16(v[k], f);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const float dlt = f[e] - mean;
+                    ss += dlt * dlt;
+                }
+            }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+        const float rstd = rsqrtf(ss * invD + 1e-6f);
+        uint4 *dst = reinterpret_cast<uint4 *>(out + (int64_t)j * D);
+#pragma unroll
+        for (int k = 0; k < CPL; ++k) {
+            const int c = lane + 32 * k;
+            if (c < C) {
+                float f[8];
+                unpack8_bf16(v[k], f);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) f[e] = (f[e] - mean) * rstd;
+                dst[c] = pack8_bf16(f);
+            }
+        }
+    }
+}
+
+template <int CPL>
+void launch_warp_bf16(const __nv_bfloat16 *in, const int32_t *rows, int n_rows, int D,
+                      __nv_bfloat16 *out, cudaStream_t st) {
+    constexpr int RPB = kThreads / 32;
+    int grid = (n_rows + RPB - 1) / RPB;
+    if (grid > 152 * 8) grid = 152 * 8;
+    layernorm_warp_bf16<CPL><<<grid, kThreads, 0, st>>>(in, rows, n_rows, D, out);
+}
+
 template <typename T>
 void launch_t(const T *in, const int32_t *rows, int n_rows, int D, __nv_bfloat16 *out,
               cudaStream_t st) {
     const int C = D / 8;
     echo::LaunchScope ls(ECHO_K_LAYERNORM, n_rows, D, 0, st);
+    if constexpr (sizeof(T) == 2) {
+        const int cpl = (C + 31) / 32;   // 16-byte chunks per lane
+        if (cpl <= 4) return launch_warp_bf16<4>(in, rows, n_rows, D, out, st);
+        if (cpl <= 8) return launch_warp_bf16<8>(in, rows, n_rows, D, out, st);
+        if (cpl <= 16) return launch_warp_bf16<16>(in, rows, n_rows, D, out, st);
+        if (cpl <= 20) return launch_warp_bf16<20>(in, rows, n_rows, D, out, st);
+        if (cpl <= 24) return launch_warp_bf16<24>(in, rows, n_rows, D, out, st);
+        return launch_warp_bf16<32>(in, rows, n_rows, D, out, st);
+    }
     if (C <= 32 * kMaxChunks / 2) {   // D <= 1024: a warp per row
         constexpr int RPB = kThreads / 32;
         int grid = (n_rows + RPB - 1) / RPB;

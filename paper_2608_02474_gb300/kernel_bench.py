@@ -23,7 +23,8 @@ from . import echocache as ec
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--kernel", required=True,
-                    choices=["gemm", "attention", "drift", "select", "merge", "quant", "layernorm"])
+                    choices=["gemm", "attention", "drift", "select", "merge", "quant", "layernorm",
+                             "energy"])
     ap.add_argument("--M", type=int, default=6552)
     ap.add_argument("--N", type=int, default=5120)
     ap.add_argument("--K", type=int, default=5120)
@@ -33,6 +34,9 @@ def main():
     ap.add_argument("--T", type=int, default=21)
     ap.add_argument("--D", type=int, default=5120)
     ap.add_argument("--act", type=int, default=0)
+    ap.add_argument("--rows", type=int, default=0, help="layernorm: gather this many rows")
+    ap.add_argument("--f32", action="store_true", help="layernorm: fp32 input")
+    ap.add_argument("--samples", type=int, default=80960, help="energy: audio samples")
     ap.add_argument("--iters", type=int, default=3)
     ap.add_argument("--warmup", type=int, default=1)
     a = ap.parse_args()
@@ -89,12 +93,21 @@ def main():
             run = lambda: ec.echo_block_step(_W, dims, x, None, 0, q, s, y=y, workspace=ws)
             work = NT * (D + 4.0) + NT * 2.0 * D + 4.0 * NT
         unit = "GB/s"
+    elif a.kernel == "energy":
+        audio = rn(a.samples)
+        band = torch.empty(a.T, 8, dtype=torch.float32, device=dev)
+        seg = torch.empty(a.T, dtype=torch.float32, device=dev)
+        run = lambda: ec.echo_audio_energy(audio, a.T, band=band, seg=seg)
+        work, unit = 4.0 * a.samples, "GB/s"
     else:  # layernorm
         NT = a.T * a.N
-        x = rn(NT, a.D).to(torch.bfloat16)
-        out = torch.empty_like(x)
-        run = lambda: ec.echo_layernorm(x, out=out)
-        work, unit = NT * 4.0 * a.D, "GB/s"
+        x = rn(NT, a.D) if a.f32 else rn(NT, a.D).to(torch.bfloat16)
+        n = a.rows if a.rows else NT
+        rows = torch.sort(torch.randperm(NT, generator=g, device=dev)[:n]).values.to(torch.int32) \
+            if a.rows else None
+        out = torch.empty(n, a.D, dtype=torch.bfloat16, device=dev)
+        run = lambda: ec.echo_layernorm(x, rows=rows, out=out)
+        work, unit = n * (x.element_size() + 2.0) * a.D, "GB/s"
 
     for _ in range(a.warmup):
         run()
