@@ -287,6 +287,23 @@ def run_reference(args, w, rnum, rden, rank):
     print(json.dumps(line), flush=True)
 
 
+def slowest_rank_ms(ms: float, world: int, device=None) -> float:
+    """The step time of the job: the maximum over ranks (replicas run in
+    lock-step between barriers, so the slowest one sets the pace)."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tokens_per_s(tokens_per_replica: int, world: int, ms: float) -> float:
+    """Whole-job throughput: every replica processes its own tokens."""
+    return world * tokens_per_replica / (ms * 1e-3)
+
+
 def run_sweep(args, w, blocks, x0, xs, dev, rank, world):
     """Cached step time for every (audio profile, ratio) and the uncached block."""
     import torch
@@ -425,13 +442,9 @@ def main():
     barrier()
     launches = ec.echo_launch_count() - l0
     clk = clocks.stop()
-    ms = ev0.elapsed_time(ev1) / args.steps
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = slowest_rank_ms(ev0.elapsed_time(ev1) / args.steps, world, dev)
     assert ec.echo_get_device_error() == 0
-    value = world * w.NT / (ms * 1e-3)
+    value = job_tokens_per_s(w.NT, world, ms)
 
     # ---- per-kernel times: the same steps again with every launch bracketed by events ----
     ec.echo_profile_enable(True)
@@ -461,12 +474,8 @@ def main():
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
-        ems = e0.elapsed_time(e1) / args.steps
-        if world > 1:
-            t = torch.tensor([ems], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ems = float(t.item())
-        e2e = {"value": round(world * w.NT / (ems * 1e-3), 2), "unit": UNIT,
+        ems = slowest_rank_ms(e0.elapsed_time(e1) / args.steps, world, dev)
+        e2e = {"value": round(job_tokens_per_s(w.NT, world, ems), 2), "unit": UNIT,
                "h2d_bytes_per_step": xh[0].numel() * 2, "d2h_bytes_per_step": yh[0].numel() * 2,
                "ms_per_step": round(ems, 3)}
 

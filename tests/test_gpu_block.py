@@ -151,15 +151,20 @@ def test_edge_ratios_and_aliasing(ec):
 
 
 @pytest.mark.slow
-def test_wan_block_sampled_rows(ec):
-    """Full-size Wan2.2-S2V-shaped block (32760 tokens, D 5120, 40 heads) at r = 1/5:
-    indices bit-exact, inactive rows bit-exact, 64 sampled active rows (32 random,
-    32 of highest score) against the oracle with keys/values over all tokens."""
-    w = WAN_BLOCK_32760
+@pytest.mark.parametrize("name,layer", [("wan_block_32760", 0), ("wan_stack40_32760", 39),
+                                        ("wan_sweep_63960", 0)])
+def test_wan_block_sampled_rows(ec, name, layer):
+    """Full-size Wan2.2-S2V-shaped blocks (D 5120, 40 heads) at r = 1/5: the
+    32760-token block, the last layer of the 40-layer stack (its own weights),
+    and the 63960-token sweep shape.  Indices bit-exact, inactive rows
+    bit-exact, 64 sampled active rows (32 random, 32 of highest score) against
+    the oracle with keys/values over all tokens."""
+    from synth import ALL
+    w = ALL[name]
     audio = G.audio(w)
     _, e = oracle.energy.audio_energy(audio, w.T)
     e32 = e.astype(F32)
-    W = G.block_weights(w, 0)
+    W = G.block_weights(w, layer)
     cond = G.cond_tokens(w, audio)
     x0 = G.latents(w)
     x1 = G.step_input(w, x0, 1)
