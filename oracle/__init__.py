@@ -16,7 +16,8 @@ Modules:
   block   - the DiT block on active latents (Q' on active, K/V on all, FFN on
             active) and the mask fusion.
   step    - one cached layer step, the step loop, the uncached block.
+  schedule - step-level Eq. 1 change and the adaptive update rate r_t.
 
 Parity status per function is stated in each module header.
 """
-from . import block, cache, energy, select, step  # noqa: F401
+from . import block, cache, energy, schedule, select, step  # noqa: F401
