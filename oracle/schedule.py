@@ -15,6 +15,7 @@ r_max, alpha.  Readings:
   * Delta-hat = Delta / Delta_ref with Delta_ref the change measured at the
     first cached step (the first Delta available after the full warm-up step),
     so Delta-hat starts at 1; a zero reference leaves Delta-hat = 0;
+  * before any change is known (the first cached step) Delta-hat = 1;
   * one global budget K = ceil(r_t * NT) (as for the fixed ratio), computed in
     fp64 and clamped to [0, NT];
   * defaults r_min = 0.1, r_max = 0.5, alpha = 0.2, xi = 1e-6.
@@ -55,3 +56,30 @@ def budget(rate: float, NT: int) -> int:
 def adaptive_budget(delta: float, delta_ref: float, NT: int, r_min: float = R_MIN,
                     r_max: float = R_MAX, alpha: float = ALPHA) -> int:
     return budget(update_rate(normalised(delta, delta_ref), r_min, r_max, alpha), NT)
+
+
+class Schedule:
+    """The step loop's state: the Eq. 1 changes seen so far and the budgets
+    handed out.  `budget()` gives the next cached step's K from the latest
+    change (Delta-hat = 1 before any is known); `observe(h_prev, h_cur)` adds
+    the change between two consecutive step outputs."""
+
+    def __init__(self, NT: int, r_min: float = R_MIN, r_max: float = R_MAX, alpha: float = ALPHA,
+                 xi: float = XI):
+        self.NT, self.r_min, self.r_max, self.alpha, self.xi = NT, r_min, r_max, alpha, xi
+        self.deltas: list[float] = []
+        self.budgets: list[int] = []
+
+    def budget(self) -> int:
+        if self.deltas:
+            K = adaptive_budget(self.deltas[-1], self.deltas[0], self.NT, self.r_min, self.r_max,
+                                self.alpha)
+        else:
+            K = budget(update_rate(1.0, self.r_min, self.r_max, self.alpha), self.NT)
+        self.budgets.append(K)
+        return K
+
+    def observe(self, h_prev: np.ndarray, h_cur: np.ndarray) -> float:
+        d = step_delta(h_prev, h_cur, self.xi)
+        self.deltas.append(d)
+        return d

@@ -7,8 +7,8 @@ latents (energy-guided), run the block on them (Q' on active, K/V on all),
 fuse with the reconstructed cache, write the active rows back into the int8
 cache.  The paper keeps full computation in the early steps; the number of
 such steps is not given.  Reading: step 0 is a full step (K = NT) that fills
-every layer's cache; later steps use the fixed ratio r (the adaptive r_t of
-the paper is not part of this path).  Layer I/O is stored as bf16 (the
+every layer's cache; later steps use the fixed ratio r, or the adaptive r_t
+of the paper (schedule.py) when a schedule is given.  Layer I/O is stored as bf16 (the
 workload's storage type): the merged output is rounded to bf16 before it feeds
 the next layer, and the cache quantises the bf16 value of y_act.
 
@@ -64,26 +64,39 @@ def cached_layer_step(x, q, s, seg_energy, W, cond, T, N, H, ratio_num, ratio_de
 
 def generation(x_inputs, weights, cond, seg_energy, T, N, H, ratio_num, ratio_den,
                lam=0.1, xi=1e-6, mode=select.MODE_ENERGY_DRIFT, warmup_steps=1,
-               record=None):
+               record=None, rate=None):
     """Step loop over len(x_inputs) steps and len(weights) layers.
 
     x_inputs[t] is the layer-0 input at step t; layer l+1 takes layer l's merged
     output.  Steps < warmup_steps are full.  `record(t, l, x, q, s, result)` is
-    called for every layer step with that step's inputs.  Returns the final
+    called for every layer step with that step's inputs.  With `rate` (a
+    schedule.Schedule) the cached steps take the adaptive budget of Sec. 3.3
+    instead of ratio_num / ratio_den: every layer of step t refreshes
+    K_t = rate.budget() tokens, and after each step rate.observe() gets the
+    last layer's output of the step before and of this one.  Returns the final
     per-layer caches."""
     NT, D = x_inputs[0].shape
     L = len(weights)
     qs = [np.zeros((NT, D), dtype=np.int8) for _ in range(L)]
     ss = [np.zeros(NT, dtype=np.float32) for _ in range(L)]
+    h_prev = None
     for t, x0 in enumerate(x_inputs):
         x = x0
+        full = t < warmup_steps
+        num, den = ratio_num, ratio_den
+        if rate is not None and not full:
+            num, den = rate.budget(), NT
         for l in range(L):
             r = cached_layer_step(x, qs[l], ss[l], seg_energy, weights[l], cond[l], T, N, H,
-                                  ratio_num, ratio_den, lam, xi, mode, full=t < warmup_steps)
+                                  num, den, lam, xi, mode, full=full)
             if record is not None:
                 record(t, l, x, qs[l], ss[l], r)
             qs[l], ss[l] = r.q, r.s
             x = r.y_bf16
+        if rate is not None:
+            if h_prev is not None:
+                rate.observe(h_prev, x)
+            h_prev = x
     return qs, ss
 
 
