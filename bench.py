@@ -44,6 +44,10 @@ def parse():
     ap.add_argument("--profile", default="audio", help="audio profile")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--adaptive", default=None, metavar="R_MIN,R_MAX,ALPHA",
+                    help="adaptive update rate (Sec. 3.3) instead of a fixed ratio, e.g. "
+                         "0.1,0.5,0.2; the change of Eq. 1 between consecutive step outputs "
+                         "and the host rule are part of every timed step")
     ap.add_argument("--sweep", action="store_true",
                     help="refresh-ratio x audio-profile sweep against the uncached block "
                          "(one JSON line per point and a break-even summary)")
@@ -119,6 +123,8 @@ def algorithmic_work(name, m, n, k, K, xbytes=2):
         return None, m * n * 3 + 8.0 * m
     if name == "layernorm_gather":
         return None, m * n * 4
+    if name == "step_delta" and m > 0:
+        return None, 2.0 * m * n
     return None, None
 
 
@@ -195,7 +201,7 @@ def load_peaks():
 
 
 # ---------------------------------------------------------------------------
-def oracle_sample(w, audio, W, cond, x1, q, s, rnum, rden, budget_s=25.0):
+def oracle_sample(w, audio, W, cond, x1, q, s, rnum, rden, budget_s=25.0, adaptive=False):
     """Time the CPU oracle on a bounded sample of one cached step and extrapolate.
 
     Measured in full: audio energy, drift + top-K over all tokens, the merge
@@ -233,10 +239,17 @@ def oracle_sample(w, audio, W, cond, x1, q, s, rnum, rden, budget_s=25.0):
     per_layer = (t["select"] + t["kv_sample"] * w.NT / s_kv + t["active_sample"] * K / s_a
                  + t["merge_quant"])
     step_s = t["energy"] + w.layers * per_layer
+    if adaptive:
+        t0 = time.perf_counter()
+        oracle.schedule.step_delta(kv_stand_in, x1)   # two [NT, D] arrays: timing only
+        t["step_delta"] = time.perf_counter() - t0
+        step_s += t["step_delta"]
     sample = (f"oracle on one {w.name} cached step: energy, drift+top-K over all {w.NT} tokens, "
               f"merge and int8 write in full; K/V projection timed on {s_kv} of {w.NT} rows and "
               f"the active-row block on {s_a} of {K} rows, each scaled to the full count; "
-              f"one layer timed, times {w.layers} layers; {sum(t.values()):.1f} s of CPU time")
+              f"one layer timed, times {w.layers} layers"
+              + ("; the step-level Eq. 1 change over all NT x D values in full" if adaptive else "")
+              + f"; {sum(t.values()):.1f} s of CPU time")
     return step_s, sample, t
 
 
@@ -390,7 +403,7 @@ def main():
     import torch
     import torch.distributed as dist
     from paper_2608_02474_gb300 import echocache as ec
-    from paper_2608_02474_gb300.pipeline import CachedStack
+    from paper_2608_02474_gb300.pipeline import AdaptiveRate, CachedStack
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
@@ -413,11 +426,19 @@ def main():
     x0_d = torch.from_numpy(x0).to(dev, torch.bfloat16)
     xs_d = [torch.from_numpy(x).to(dev, torch.bfloat16) for x in xs]
     stack.set_audio(audio_d)
-    stack.step(x0_d, 1, 1, full=True)          # fills every layer's cache (untimed setup)
+    rate = None
+    if args.adaptive:
+        r_min, r_max, alpha = (float(v) for v in args.adaptive.split(","))
+        rate = AdaptiveRate(w.NT, r_min, r_max, alpha, device=dev)
+        stack.step_adaptive(x0_d, rate, full=True)   # fills every layer's cache (untimed setup)
+    else:
+        stack.step(x0_d, 1, 1, full=True)          # fills every layer's cache (untimed setup)
     K = w.K if (rnum, rden) == (w.ratio_num, w.ratio_den) else (rnum * w.NT + rden - 1) // rden
 
     def one_step(x):
         stack.set_audio(audio_d)
+        if rate is not None:
+            return stack.step_adaptive(x, rate)
         return stack.step(x, rnum, rden)
 
     for i in range(args.warmup):
@@ -442,6 +463,9 @@ def main():
     barrier()
     launches = ec.echo_launch_count() - l0
     clk = clocks.stop()
+    if rate is not None:
+        timed_budgets = rate.budgets[-args.steps:]
+        K = round(sum(timed_budgets) / len(timed_budgets))
     ms = slowest_rank_ms(ev0.elapsed_time(ev1) / args.steps, world, dev)
     assert ec.echo_get_device_error() == 0
     value = job_tokens_per_s(w.NT, world, ms)
@@ -464,13 +488,14 @@ def main():
     if not args.no_e2e:
         xh = [torch.from_numpy(x).to(torch.bfloat16).pin_memory() for x in xs]
         yh = [torch.empty(w.NT, w.D, dtype=torch.bfloat16).pin_memory() for _ in range(2)]
-        stack.run_host([xh[0], xh[1]], yh, rnum, rden, audio=audio_d)
+        stack.run_host([xh[0], xh[1]], yh, rnum, rden, audio=audio_d, rate=rate)
         torch.cuda.synchronize()
         barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         stack.run_host([xh[i % 2] for i in range(args.steps)],
-                       [yh[i % 2] for i in range(args.steps)], rnum, rden, audio=audio_d)
+                       [yh[i % 2] for i in range(args.steps)], rnum, rden, audio=audio_d,
+                       rate=rate)
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
@@ -483,7 +508,9 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
         q, s, _ = oracle.cache.quantize_rows(x0)
-        step_s, sample, _ = oracle_sample(w, audio, W, cond, xs[0], q, s, rnum, rden)
+        cr = (K, w.NT) if rate is not None else (rnum, rden)
+        step_s, sample, _ = oracle_sample(w, audio, W, cond, xs[0], q, s, *cr,
+                                          adaptive=rate is not None)
         cpu = {"value": round(w.NT / step_s, 2), "unit": UNIT, "cores": cpu_cores(),
                "kind": "oracle", "sample": sample, "ms_per_step": round(step_s * 1e3, 1)}
 
@@ -493,12 +520,19 @@ def main():
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": "bf16", "data": "synthetic",
                 "config": {"workload": w.name, "tokens": w.NT, "active_tokens": K,
-                           "ratio": f"{rnum}/{rden}", "D": w.D, "heads": f"{w.H}x{w.d}",
+                           "ratio": f"{rnum}/{rden}" if rate is None else "adaptive",
+                           "D": w.D, "heads": f"{w.H}x{w.d}",
                            "ffn": w.F, "audio_tokens": w.Lc, "layers": w.layers,
                            "audio": args.profile, "parallelism": f"replicas{world}",
                            "l2": "inputs larger than L2 (x 335 MB, weights 702 MB per block)"},
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
                 "gpu_launches": launches, "kernels": table}
+        if rate is not None:
+            line["config"]["adaptive"] = {
+                "r_min": rate.r_min, "r_max": rate.r_max, "alpha": rate.alpha,
+                "timed_budgets": timed_budgets,
+                "note": "active_tokens = mean budget of the timed steps; each step reads back "
+                        "the change of the step before (one host synchronisation per step)"}
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()

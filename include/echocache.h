@@ -184,6 +184,45 @@ echo_status echo_select_static(const void *x, echo_dtype xt, const int8_t *cache
                                int32_t ratio_den, const echo_select_params *p,
                                int32_t *idx, int32_t *K_out, echo_stream_t stream);
 
+/* ---- step-level adaptive update rate (Sec. 3.3, with Eq. 1 of Sec. 3.1) ---- */
+
+/* Parameters of r_t = clip(r_min + alpha * Delta-hat_t, r_min, r_max); the
+ * paper gives none of the values (0 <= r_min <= r_max <= 1, alpha >= 0). */
+typedef struct {
+    double r_min;
+    double r_max;
+    double alpha;
+} echo_rate_params;
+
+/* Bytes of device workspace echo_step_delta needs (a fixed 9.5 KiB). */
+size_t echo_step_delta_workspace_size(int64_t n);
+
+/* Eq. 1 on two consecutive step outputs h_prev = h_t, h_cur = h_{t+1}:
+ *   out[1] = sum_i |h_prev[i] - h_cur[i]|,  out[2] = sum_i |h_cur[i]|,
+ *   out[0] = Delta = out[1] / (out[2] + xi),  all fp64.
+ *   h_prev, h_cur: n elements of dtype ht (bf16 or f32), device, 16-byte
+ *   aligned (may be NULL when n = 0); n >= 0 (n = 0 gives 0).  out: device double[3], written on the
+ *   stream.  workspace >= echo_step_delta_workspace_size(n) bytes, 16-byte
+ *   aligned, device, contents ignored.  Each element's difference and absolute
+ *   value are taken in fp32; the sums are compensated, so their relative error
+ *   is a few units of 2^-24; the order of summation depends on n only, so equal
+ *   inputs give equal bits on every run.
+ * Errors: INVALID_ARG (null, misaligned, xi <= 0), SHAPE (n < 0), WORKSPACE,
+ * CUDA; a non-finite Delta sets the NONFINITE device flag. */
+echo_status echo_step_delta(const void *h_prev, const void *h_cur, echo_dtype ht, int64_t n,
+                            double xi, double *out, void *workspace, size_t ws_bytes,
+                            echo_stream_t stream);
+
+/* Host function (no GPU work): the step's update rate and budget from Eq. 1's
+ * step-level change, Delta-hat = delta / delta_ref (0 when delta_ref == 0):
+ *   *rate = min(max(r_min + alpha * Delta-hat, r_min), r_max)
+ *   *K    = min(max(ceil(*rate * NT), 0), NT)   (k_t = ceil(N r_t), one global budget)
+ * every operation in fp64 with one rounding each, in the order written.
+ * rate may be NULL.  Errors: INVALID_ARG (parameters), SHAPE (NT < 0),
+ * NONFINITE (delta or delta_ref negative or not finite). */
+echo_status echo_update_rate(double delta, double delta_ref, const echo_rate_params *p,
+                             int32_t NT, double *rate, int32_t *K);
+
 /* Bytes of workspace echo_block_step needs for dims and up to K_max active
  * tokens (also enough for echo_precompute_cross_kv). */
 size_t echo_workspace_size(const echo_block_dims *dims, int32_t K_max);
@@ -273,7 +312,7 @@ echo_status echo_layernorm(const void *in, echo_dtype in_t, const int32_t *rows,
 typedef enum {
     ECHO_K_ENERGY = 0, ECHO_K_DRIFT = 1, ECHO_K_TOPK = 2, ECHO_K_ROWMAP = 3,
     ECHO_K_LAYERNORM = 4, ECHO_K_GEMM = 5, ECHO_K_ATTENTION = 6, ECHO_K_QUANT = 7,
-    ECHO_K_DEQUANT = 8, ECHO_K_MERGE = 9, ECHO_K_COUNT = 10
+    ECHO_K_DEQUANT = 8, ECHO_K_MERGE = 9, ECHO_K_STEP_DELTA = 10, ECHO_K_COUNT = 11
 } echo_kernel_kind;
 
 /* Number of kernels this library has launched in this process (all devices). */
@@ -289,7 +328,8 @@ echo_status echo_profile_enable(int32_t on);
  * the host arrays, clears the record list and returns the number copied (or
  * -1 on a CUDA error).  Shapes: GEMM (M, N, Kd); ATTENTION (M queries, L keys,
  * H * d); DRIFT (NT, D, 0); TOPK (NT, K, 0); LAYERNORM, QUANT, DEQUANT,
- * MERGE (rows, D, 0); ENERGY (T, frames, n_fft). */
+ * MERGE (rows, D, 0); ENERGY (T, frames, n_fft); STEP_DELTA (n, element bytes, 0)
+ * for the reduction and (0, 0, blocks) for its final combine. */
 int32_t echo_profile_read(int32_t max, int32_t *kinds, int64_t *m, int64_t *n, int64_t *k,
                           float *ms);
 

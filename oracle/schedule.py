@@ -33,11 +33,18 @@ import numpy as np
 R_MIN, R_MAX, ALPHA, XI = 0.1, 0.5, 0.2, 1e-6
 
 
+def step_sums(h_prev: np.ndarray, h_cur: np.ndarray) -> tuple[float, float]:
+    """The two L1 norms of Eq. 1, ||h_prev - h_cur||_1 and ||h_cur||_1, as fp64
+    sums of the exact inputs."""
+    a = np.asarray(h_prev, dtype=np.float64).ravel()
+    b = np.asarray(h_cur, dtype=np.float64).ravel()
+    return float(np.abs(a - b).sum()), float(np.abs(b).sum())
+
+
 def step_delta(h_prev: np.ndarray, h_cur: np.ndarray, xi: float = XI) -> float:
-    """Eq. 1 on two consecutive step outputs, fp64 sums of the exact inputs."""
-    a = np.asarray(h_prev, dtype=np.float64)
-    b = np.asarray(h_cur, dtype=np.float64)
-    return float(np.abs(a - b).sum() / (np.abs(b).sum() + xi))
+    """Eq. 1 on two consecutive step outputs."""
+    num, den = step_sums(h_prev, h_cur)
+    return num / (den + xi)
 
 
 def normalised(delta: float, delta_ref: float) -> float:

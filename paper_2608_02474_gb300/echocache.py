@@ -22,6 +22,7 @@ MODE_ENERGY_DRIFT, MODE_SEGMENT, MODE_DRIFT_ONLY = 0, 1, 2
 
 _c = ctypes
 _vp, _i32, _i64, _sz, _f32 = _c.c_void_p, _c.c_int32, _c.c_int64, _c.c_size_t, _c.c_float
+_f64 = _c.c_double
 
 
 class EchoError(RuntimeError):
@@ -32,6 +33,10 @@ class EchoError(RuntimeError):
 
 class SelectParams(_c.Structure):
     _fields_ = [("lambda_", _f32), ("xi", _f32), ("mode", _i32)]
+
+
+class RateParams(_c.Structure):
+    _fields_ = [("r_min", _f64), ("r_max", _f64), ("alpha", _f64)]
 
 
 class BlockDims(_c.Structure):
@@ -53,6 +58,10 @@ _SIGS = {
                            _c.POINTER(SelectParams), _vp, _c.POINTER(_i32), _vp, _vp, _sz, _vp]),
     "echo_select_static": (_i32, [_vp, _i32, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32,
                                   _c.POINTER(SelectParams), _vp, _c.POINTER(_i32), _vp]),
+    "echo_step_delta_workspace_size": (_sz, [_i64]),
+    "echo_step_delta": (_i32, [_vp, _vp, _i32, _i64, _f64, _vp, _vp, _sz, _vp]),
+    "echo_update_rate": (_i32, [_f64, _f64, _c.POINTER(RateParams), _i32, _c.POINTER(_f64),
+                                _c.POINTER(_i32)]),
     "echo_workspace_size": (_sz, [_c.POINTER(BlockDims), _i32]),
     "echo_precompute_cross_kv": (_i32, [_vp, _vp, _vp, _i32, _i32, _vp, _vp]),
     "echo_block_step": (_i32, [_c.POINTER(BlockWeightsC), _c.POINTER(BlockDims), _vp, _vp, _i32,
@@ -157,6 +166,39 @@ def echo_select(x, cache_q, cache_scale, seg_energy, T: int, N: int, ratio_num: 
         ratio_den, _c.byref(prm), _p(idx), _c.byref(K), _p(scores), _p(workspace), ws_bytes,
         _stream(stream)))
     return idx[:K.value], K.value, scores
+
+
+def echo_step_delta_workspace_size(n: int) -> int:
+    return lib().echo_step_delta_workspace_size(n)
+
+
+def echo_step_delta(h_prev, h_cur, xi: float = 1e-6, out=None, workspace=None, stream=None):
+    """Eq. 1 between two step outputs; returns the device double[3]
+    {Delta, sum|h_prev - h_cur|, sum|h_cur|} (no host synchronisation)."""
+    _dev(h_prev, "h_prev")
+    _dev(h_cur, "h_cur")
+    if h_prev.dtype != h_cur.dtype or h_prev.numel() != h_cur.numel():
+        raise ValueError("h_prev and h_cur must have the same dtype and size")
+    n = h_cur.numel()
+    out = out if out is not None else torch.empty(3, dtype=torch.float64, device=h_cur.device)
+    ws_n = echo_step_delta_workspace_size(n)
+    ws = workspace if workspace is not None else torch.empty(ws_n, dtype=torch.uint8,
+                                                             device=h_cur.device)
+    _check("echo_step_delta", lib().echo_step_delta(
+        _p(h_prev), _p(h_cur), _dtype(h_cur), n, float(xi), _p(out), _p(ws), ws.numel(),
+        _stream(stream)))
+    return out
+
+
+def echo_update_rate(delta: float, delta_ref: float, NT: int, r_min: float = 0.1,
+                     r_max: float = 0.5, alpha: float = 0.2) -> tuple[float, int]:
+    """Host rule of the adaptive update rate: returns (r_t, K)."""
+    prm = RateParams(r_min, r_max, alpha)
+    rate, K = _f64(0.0), _i32(0)
+    _check("echo_update_rate", lib().echo_update_rate(float(delta), float(delta_ref),
+                                                      _c.byref(prm), NT, _c.byref(rate),
+                                                      _c.byref(K)))
+    return rate.value, K.value
 
 
 def echo_workspace_size(dims: BlockDims, K_max: int) -> int:

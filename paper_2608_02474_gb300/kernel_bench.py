@@ -4,6 +4,7 @@
     python -m paper_2608_02474_gb300.kernel_bench --kernel attention --M 6552 --L 32760 --H 40 --d 128
     python -m paper_2608_02474_gb300.kernel_bench --kernel drift --T 21 --N 1560 --D 5120
     python -m paper_2608_02474_gb300.kernel_bench --kernel merge --T 21 --N 1560 --D 5120 --K 6552
+    python -m paper_2608_02474_gb300.kernel_bench --kernel step_delta --T 21 --N 1560 --D 5120
 
 Inputs are seeded random device tensors of the right shapes (values do not
 change the work of these kernels).  Prints the mean time per launch over
@@ -24,7 +25,7 @@ def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--kernel", required=True,
                     choices=["gemm", "attention", "drift", "select", "merge", "quant", "layernorm",
-                             "energy"])
+                             "energy", "step_delta"])
     ap.add_argument("--M", type=int, default=6552)
     ap.add_argument("--N", type=int, default=5120)
     ap.add_argument("--K", type=int, default=5120)
@@ -93,6 +94,14 @@ def main():
             run = lambda: ec.echo_block_step(_W, dims, x, None, 0, q, s, y=y, workspace=ws)
             work = NT * (D + 4.0) + NT * 2.0 * D + 4.0 * NT
         unit = "GB/s"
+    elif a.kernel == "step_delta":
+        n = a.T * a.N * a.D
+        hp = rn(n).to(torch.bfloat16)
+        hc = (hp.float() + 0.05 * rn(n)).to(torch.bfloat16)
+        out = torch.empty(3, dtype=torch.float64, device=dev)
+        ws = torch.empty(ec.echo_step_delta_workspace_size(n), dtype=torch.uint8, device=dev)
+        run = lambda: ec.echo_step_delta(hp, hc, out=out, workspace=ws)
+        work, unit = 4.0 * n, "GB/s"
     elif a.kernel == "energy":
         audio = rn(a.samples)
         band = torch.empty(a.T, 8, dtype=torch.float32, device=dev)

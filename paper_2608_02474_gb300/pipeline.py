@@ -5,13 +5,64 @@ buffers on the device and runs one denoising step as the paper orders it
 (Sec. 3.3): the audio energy once per generation, then per layer the
 energy-guided selection and the block on the selected latents.  Step 0 (or
 any step with full=True) refreshes every token and fills the caches.  No host
-synchronisation happens inside a step: K follows from the ratio on the host.
+synchronisation happens inside a fixed-ratio step: K follows from the ratio on
+the host.  An adaptive step (AdaptiveRate) reads one scalar back: the change
+of the step before.
 """
 from __future__ import annotations
 
 import torch
 
 from . import echocache as ec
+
+
+class AdaptiveRate:
+    """The step-level update rate of Sec. 3.3 for a CachedStack.
+
+    After every step the change of Eq. 1 between the stack output of that step
+    and of the step before is reduced on the device (echo_step_delta) and
+    copied into pinned host memory.  The next cached step's budget
+    (echo_update_rate) waits for that copy only: r_t follows the most recent
+    change, normalised by the first change measured (Delta-hat = 1 before any
+    change is known), and K_t = ceil(r_t NT).  Waiting for the copy is the one
+    host synchronisation of an adaptive step."""
+
+    def __init__(self, NT: int, r_min: float = 0.1, r_max: float = 0.5, alpha: float = 0.2,
+                 xi: float = 1e-6, device="cuda"):
+        self.NT, self.r_min, self.r_max, self.alpha, self.xi = NT, r_min, r_max, alpha, xi
+        dev = torch.device(device)
+        self.out = torch.zeros(3, dtype=torch.float64, device=dev)
+        self.host = torch.zeros(3, dtype=torch.float64).pin_memory()
+        self.ws = torch.empty(ec.echo_step_delta_workspace_size(0), dtype=torch.uint8, device=dev)
+        self.ready = torch.cuda.Event()
+        self.pending = False
+        self.h_prev = None
+        self.deltas: list[float] = []
+        self.rates: list[float] = []
+        self.budgets: list[int] = []
+
+    def budget(self) -> int:
+        """K for the next cached step (waits for the last change's copy)."""
+        if self.pending:
+            self.ready.synchronize()
+            self.deltas.append(float(self.host[0]))
+            self.pending = False
+        d, ref = (self.deltas[-1], self.deltas[0]) if self.deltas else (1.0, 1.0)
+        rate, K = ec.echo_update_rate(d, ref, self.NT, self.r_min, self.r_max, self.alpha)
+        self.rates.append(rate)
+        self.budgets.append(K)
+        return K
+
+    def observe(self, h_cur: torch.Tensor):
+        """Enqueue the change between the previous step's output and h_cur on
+        the current stream.  The previous output must stay unchanged until
+        this work has run."""
+        if self.h_prev is not None:
+            ec.echo_step_delta(self.h_prev, h_cur, self.xi, out=self.out, workspace=self.ws)
+            self.host.copy_(self.out, non_blocking=True)
+            self.ready.record()
+            self.pending = True
+        self.h_prev = h_cur
 
 
 class CachedStack:
@@ -67,16 +118,37 @@ class CachedStack:
             cur = dst
         return cur
 
+    def step_adaptive(self, x: torch.Tensor, rate: AdaptiveRate, full: bool = False,
+                      keep_scores: bool = False, out: torch.Tensor | None = None) -> torch.Tensor:
+        """One step whose budget follows the adaptive update rate (Sec. 3.3):
+        every layer refreshes K_t = rate.budget() tokens (all on a full step),
+        then the step's change from the previous output is enqueued.  Without
+        `out` the output alternates between two buffers of the stack, so the
+        previous output stays intact; a caller passing `out` keeps the previous
+        step's output unchanged until this step's work has run."""
+        K = self.NT if full else rate.budget()
+        if out is None:
+            if not hasattr(self, "_h"):
+                self._h = [torch.empty(self.NT, self.D, dtype=torch.bfloat16,
+                                       device=self.seg.device) for _ in range(2)]
+                self._h_i = 0
+            out = self._h[self._h_i]
+            self._h_i ^= 1
+        y = self.step(x, K, self.NT, full=full, keep_scores=keep_scores, out=out)
+        rate.observe(y)
+        return y
+
     def run_host(self, host_x: list, host_y: list, ratio_num: int, ratio_den: int,
-                 audio: torch.Tensor | None = None):
+                 audio: torch.Tensor | None = None, rate: AdaptiveRate | None = None):
         """Steps whose inputs and outputs live in pinned host memory.
 
         Step i copies host_x[i] to the device, runs one step (the audio energy
         first when `audio` is given) and copies the result into host_y[i].  The
         copies run on their own streams into double-buffered device tensors, so
         the upload of step i+1 and the download of step i-1 overlap step i.
-        Returns after everything has been enqueued; synchronise before reading
-        host_y."""
+        With `rate` every step takes the adaptive budget (ratio_num and
+        ratio_den are then unused).  Returns after everything has been
+        enqueued; synchronise before reading host_y."""
         dev = self.seg.device
         comp = torch.cuda.current_stream(dev)
         if not hasattr(self, "_h2d"):
@@ -102,7 +174,10 @@ class CachedStack:
             comp.wait_event(ev["y_copied"][b])
             if audio is not None:
                 self.set_audio(audio)
-            self.step(self._xd[b], ratio_num, ratio_den, out=self._yd[b])
+            if rate is not None:
+                self.step_adaptive(self._xd[b], rate, out=self._yd[b])
+            else:
+                self.step(self._xd[b], ratio_num, ratio_den, out=self._yd[b])
             ev["x_used"][b].record(comp)
             ev["y_ready"][b].record(comp)
             with torch.cuda.stream(self._d2h):

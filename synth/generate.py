@@ -146,3 +146,14 @@ def random_energy(T: int, seed: int, distinct: bool = True) -> np.ndarray:
         e = g.permutation(T).astype(np.float32) + np.float32(1.0)
         return (e * np.float32(0.37)).astype(np.float32)
     return g.uniform(0.1, 3.0, size=T).astype(np.float32)
+
+
+def step_output_pair(n: int, seed: int, change: float = 0.05, bf16: bool = True):
+    """Two flat length-n outputs of consecutive steps: h_prev ~ N(0, 1) and
+    h_cur = h_prev + N(0, change^2), both rounded to bf16 values when bf16."""
+    g = rng(seed)
+    a = g.standard_normal(n, dtype=np.float32)
+    b = a + g.standard_normal(n, dtype=np.float32) * np.float32(change)
+    if bf16:
+        return to_bf16_values(a), to_bf16_values(b)
+    return a, b

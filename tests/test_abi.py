@@ -124,3 +124,42 @@ def test_kernel_entry_points_check_shapes(ec):
     assert L.echo_audio_energy(_vp(FAKE), 16000, 4, 500, 160, 8, _vp(FAKE), _vp(FAKE), None) == 2
     # zero rows are a no-op
     assert L.echo_cache_quant(None, 0, None, 0, 64, None, None, None) == 0
+
+
+def test_step_delta_argument_checks(ec):
+    L = ec.lib()
+    out = ctypes.c_void_p(FAKE)
+    ws = ec.echo_step_delta_workspace_size(1 << 20)
+    assert ws >= 16
+    call = lambda a=FAKE, n=1024, xi=1e-6, wsb=ws, o=FAKE, dt=0: L.echo_step_delta(
+        _vp(a), _vp(FAKE), dt, n, xi, _vp(o), _vp(FAKE), wsb, None)
+    assert call(a=0) == 1                      # null input
+    assert call(a=FAKE + 2) == 1               # misaligned
+    assert call(o=FAKE + 4) == 1               # misaligned double output
+    assert call(dt=5) == 1                     # unknown dtype
+    assert call(xi=0.0) == 1                   # xi must be > 0
+    assert call(n=-1) == 2
+    assert call(wsb=ws - 1) == 3
+
+
+def test_update_rate_rule_is_the_oracle_rule(ec):
+    """echo_update_rate is host arithmetic: its rate and budget are those of the
+    oracle's rule for the same change, bit for bit."""
+    import numpy as np
+    from oracle import schedule as S
+    rs = np.random.default_rng(11)
+    for _ in range(20000):
+        d, ref = float(rs.uniform(0, 3)), float(rs.choice([0.0, rs.uniform(1e-3, 2)]))
+        NT = int(rs.choice([0, 1, 256, 7800, 32760, 63960]))
+        r_min = float(rs.choice([0.0, 0.05, 0.1]))
+        r_max, alpha = float(rs.choice([0.3, 0.5, 1.0])), float(rs.choice([0.0, 0.2, 0.35, 1e6]))
+        rate, K = ec.echo_update_rate(d, ref, NT, r_min, r_max, alpha)
+        assert rate == S.update_rate(S.normalised(d, ref), r_min, r_max, alpha)
+        assert K == S.adaptive_budget(d, ref, NT, r_min, r_max, alpha)
+    # the clip and the first cached step (Delta-hat = 1)
+    assert ec.echo_update_rate(0.0, 1.0, 100) == (0.1, 10)
+    assert ec.echo_update_rate(9.0, 1.0, 100) == (0.5, 50)
+    with pytest.raises(ec.EchoError):
+        ec.echo_update_rate(float("nan"), 1.0, 100)
+    with pytest.raises(ec.EchoError):
+        ec.echo_update_rate(0.1, 1.0, 100, r_min=0.6, r_max=0.5)

@@ -19,6 +19,12 @@ def test_delta_of_scaled_output_closed_form(c):
                                                           rel=1e-12)
 
 
+def test_sums_on_a_worked_example():
+    # |1-2| + |-2-2| + |3+1| = 9 and |2| + |2| + |-1| = 5
+    assert S.step_sums(np.array([1.0, -2.0, 3.0]), np.array([2.0, 2.0, -1.0])) == (9.0, 5.0)
+    assert S.step_delta(np.array([1.0, -2.0, 3.0]), np.array([2.0, 2.0, -1.0]), xi=1.0) == 1.5
+
+
 def test_delta_of_zero_pair_and_from_zero():
     z = np.zeros((4, 8))
     h = G.random_rows(4, 8, seed=3).astype(np.float64)
