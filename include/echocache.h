@@ -184,6 +184,24 @@ echo_status echo_select_static(const void *x, echo_dtype xt, const int8_t *cache
                                int32_t ratio_den, const echo_select_params *p,
                                int32_t *idx, int32_t *K_out, echo_stream_t stream);
 
+/* ---- ablation selections (Sec. 4, Table 2: "Uniform" and "Random" in place
+ *      of the energy-guided anchor selection); no energy and no drift ---- */
+
+/* K = ceil(ratio_num T N / ratio_den) tokens evenly spaced over the token
+ * order: idx[j] = floor(j T N / K), ascending and distinct.  idx int32 [K]
+ * device, 16-byte aligned; *K_out (host) = K.  Errors: INVALID_ARG, SHAPE, CUDA. */
+echo_status echo_select_uniform(int32_t T, int32_t N, int32_t ratio_num, int32_t ratio_den,
+                                int32_t *idx, int32_t *K_out, echo_stream_t stream);
+
+/* The K = ceil(ratio_num T N / ratio_den) tokens with the largest keys (key
+ * descending, index ascending), as an ascending index list.  keys f32 [T N]
+ * device, drawn by the caller (independent uniform keys give a uniformly
+ * random K-subset); finite values.  idx int32 [K] device.  *K_out (host) = K.
+ * Errors: INVALID_ARG, SHAPE, CUDA. */
+echo_status echo_select_random(const float *keys, int32_t T, int32_t N, int32_t ratio_num,
+                               int32_t ratio_den, int32_t *idx, int32_t *K_out,
+                               echo_stream_t stream);
+
 /* ---- step-level adaptive update rate (Sec. 3.3, with Eq. 1 of Sec. 3.1) ---- */
 
 /* Parameters of r_t = clip(r_min + alpha * Delta-hat_t, r_min, r_max); the
@@ -312,7 +330,8 @@ echo_status echo_layernorm(const void *in, echo_dtype in_t, const int32_t *rows,
 typedef enum {
     ECHO_K_ENERGY = 0, ECHO_K_DRIFT = 1, ECHO_K_TOPK = 2, ECHO_K_ROWMAP = 3,
     ECHO_K_LAYERNORM = 4, ECHO_K_GEMM = 5, ECHO_K_ATTENTION = 6, ECHO_K_QUANT = 7,
-    ECHO_K_DEQUANT = 8, ECHO_K_MERGE = 9, ECHO_K_STEP_DELTA = 10, ECHO_K_COUNT = 11
+    ECHO_K_DEQUANT = 8, ECHO_K_MERGE = 9, ECHO_K_STEP_DELTA = 10, ECHO_K_UNIFORM = 11,
+    ECHO_K_COUNT = 12
 } echo_kernel_kind;
 
 /* Number of kernels this library has launched in this process (all devices). */
@@ -329,7 +348,7 @@ echo_status echo_profile_enable(int32_t on);
  * -1 on a CUDA error).  Shapes: GEMM (M, N, Kd); ATTENTION (M queries, L keys,
  * H * d); DRIFT (NT, D, 0); TOPK (NT, K, 0); LAYERNORM, QUANT, DEQUANT,
  * MERGE (rows, D, 0); ENERGY (T, frames, n_fft); STEP_DELTA (n, element bytes, 0)
- * for the reduction and (0, 0, blocks) for its final combine. */
+ * for the reduction and (0, 0, blocks) for its final combine; UNIFORM (NT, K, 0). */
 int32_t echo_profile_read(int32_t max, int32_t *kinds, int64_t *m, int64_t *n, int64_t *k,
                           float *ms);
 

@@ -29,9 +29,14 @@ score_i = w_{floor(i/N)} * d_i (fp32); the K tokens with the largest key
 list (the compact form of the mask).  Mode SEGMENT is the paper-literal anchor:
 d_i = 1 and lam = 0, so whole high-energy segments fill the budget in index order.
 
+The ablation selections of Sec. 4 (Uniform, Random) take neither energy nor
+drift: `uniform` spaces K tokens evenly, `random_subset` takes the top K of
+keys the caller draws.
+
 Pins: brute force over all subsets on tiny inputs, a full sort, r = 0 / r = 1,
 x == c gives 0, the canonical order on hand-built cases where order matters,
-an fp32 error bound against the exact sum.
+an fp32 error bound against the exact sum; uniform spacing by counting,
+random subsets by the brute-force top-K and by frequency.
 """
 from __future__ import annotations
 
@@ -112,6 +117,21 @@ def top_k(score: np.ndarray, K: int) -> np.ndarray:
     NT = score.shape[0]
     order = np.lexsort((np.arange(NT), -score.astype(np.float64)))
     return np.sort(order[:K]).astype(np.int32)
+
+
+def uniform(NT: int, K: int) -> np.ndarray:
+    """Uniform selection (the "Uniform" ablation of Sec. 4, Table 2): K tokens
+    evenly spaced over the token order, idx_j = floor(j NT / K), integers only."""
+    if K <= 0:
+        return np.zeros(0, dtype=np.int32)
+    return (np.arange(K, dtype=np.int64) * NT // K).astype(np.int32)
+
+
+def random_subset(keys: np.ndarray, K: int) -> np.ndarray:
+    """Random selection (the "Random" ablation of Sec. 4, Table 2): the K tokens
+    with the largest caller-drawn keys (key desc, index asc); with keys drawn
+    independently and uniformly this is a uniformly random K-subset."""
+    return top_k(np.asarray(keys, dtype=np.float32), K)
 
 
 def select(x, q, s, seg_energy, T: int, N: int, ratio_num: int, ratio_den: int,

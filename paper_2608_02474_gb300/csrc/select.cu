@@ -266,6 +266,12 @@ topk_kernel(const float *__restrict__ scores, int NT, int K, int keys_in_smem,
 
 size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
 
+// idx[j] = floor(j NT / K): K evenly spaced tokens, ascending and distinct
+__global__ void uniform_kernel(int NT, int K, int32_t *__restrict__ idx) {
+    for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < K; j += gridDim.x * blockDim.x)
+        idx[j] = (int32_t)(((int64_t)j * NT) / K);
+}
+
 }  // namespace
 
 extern "C" size_t echo_select_workspace_size(int32_t T, int32_t N) {
@@ -423,6 +429,62 @@ extern "C" echo_status echo_select_static(const void *x, echo_dtype xt, const in
     {
         LaunchScope ls(ECHO_K_TOPK, NT, K, 0, st);
         topk_kernel<<<1, kTopkThreads, dyn, st>>>(sc, NT, K, in_smem, idx);
+    }
+    return last_launch_status();
+}
+
+namespace {
+
+// shared argument checks of the ablation selections; returns K or -1
+int ablation_budget(int32_t T, int32_t N, int32_t ratio_num, int32_t ratio_den) {
+    if (T < 1 || N < 1 || ratio_den < 1 || ratio_num < 0 || ratio_num > ratio_den) return -1;
+    const int64_t NT64 = (int64_t)T * N;
+    if (NT64 > (int64_t)INT32_MAX / 2) return -1;
+    return (int)(((int64_t)ratio_num * NT64 + ratio_den - 1) / ratio_den);
+}
+
+}  // namespace
+
+extern "C" echo_status echo_select_uniform(int32_t T, int32_t N, int32_t ratio_num,
+                                           int32_t ratio_den, int32_t *idx, int32_t *K_out,
+                                           echo_stream_t stream) {
+    using namespace echo;
+    if (!idx || !K_out || !aligned16(idx)) return ECHO_ERR_INVALID_ARG;
+    const int K = ablation_budget(T, N, ratio_num, ratio_den);
+    if (K < 0) return ECHO_ERR_SHAPE;
+    if (!device_supported()) return ECHO_ERR_UNSUPPORTED;
+    *K_out = K;
+    if (K == 0) return ECHO_OK;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const int grid = (K + 255) / 256;
+    {
+        LaunchScope ls(ECHO_K_UNIFORM, T * N, K, 0, st);
+        uniform_kernel<<<grid, 256, 0, st>>>(T * N, K, idx);
+    }
+    return last_launch_status();
+}
+
+extern "C" echo_status echo_select_random(const float *keys, int32_t T, int32_t N,
+                                          int32_t ratio_num, int32_t ratio_den, int32_t *idx,
+                                          int32_t *K_out, echo_stream_t stream) {
+    using namespace echo;
+    if (!keys || !idx || !K_out || !aligned16(keys) || !aligned16(idx)) return ECHO_ERR_INVALID_ARG;
+    const int K = ablation_budget(T, N, ratio_num, ratio_den);
+    if (K < 0) return ECHO_ERR_SHAPE;
+    if (!device_supported()) return ECHO_ERR_UNSUPPORTED;
+    *K_out = K;
+    const int NT = T * N;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const size_t key_bytes = (size_t)NT * sizeof(uint32_t);
+    const int in_smem = key_bytes <= 200 * 1024 ? 1 : 0;
+    const size_t dyn = in_smem ? key_bytes : 0;
+    if (dyn > 48 * 1024 &&
+        cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn) !=
+            cudaSuccess)
+        return ECHO_ERR_CUDA;
+    {
+        LaunchScope ls(ECHO_K_TOPK, NT, K, 0, st);
+        topk_kernel<<<1, kTopkThreads, dyn, st>>>(keys, NT, K, in_smem, idx);
     }
     return last_launch_status();
 }

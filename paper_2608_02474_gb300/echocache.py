@@ -58,6 +58,8 @@ _SIGS = {
                            _c.POINTER(SelectParams), _vp, _c.POINTER(_i32), _vp, _vp, _sz, _vp]),
     "echo_select_static": (_i32, [_vp, _i32, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32,
                                   _c.POINTER(SelectParams), _vp, _c.POINTER(_i32), _vp]),
+    "echo_select_uniform": (_i32, [_i32, _i32, _i32, _i32, _vp, _c.POINTER(_i32), _vp]),
+    "echo_select_random": (_i32, [_vp, _i32, _i32, _i32, _i32, _vp, _c.POINTER(_i32), _vp]),
     "echo_step_delta_workspace_size": (_sz, [_i64]),
     "echo_step_delta": (_i32, [_vp, _vp, _i32, _i64, _f64, _vp, _vp, _sz, _vp]),
     "echo_update_rate": (_i32, [_f64, _f64, _c.POINTER(RateParams), _i32, _c.POINTER(_f64),
@@ -166,6 +168,28 @@ def echo_select(x, cache_q, cache_scale, seg_energy, T: int, N: int, ratio_num: 
         ratio_den, _c.byref(prm), _p(idx), _c.byref(K), _p(scores), _p(workspace), ws_bytes,
         _stream(stream)))
     return idx[:K.value], K.value, scores
+
+
+def echo_select_uniform(T: int, N: int, ratio_num: int, ratio_den: int, idx=None, device=None,
+                        stream=None):
+    """Uniform ablation selection; returns (idx[:K], K)."""
+    dev = idx.device if idx is not None else (device or torch.device("cuda"))
+    idx = idx if idx is not None else torch.empty(T * N, dtype=torch.int32, device=dev)
+    K = _i32(0)
+    _check("echo_select_uniform", lib().echo_select_uniform(T, N, ratio_num, ratio_den, _p(idx),
+                                                            _c.byref(K), _stream(stream)))
+    return idx[:K.value], K.value
+
+
+def echo_select_random(keys, T: int, N: int, ratio_num: int, ratio_den: int, idx=None,
+                       stream=None):
+    """Random ablation selection over caller-drawn keys; returns (idx[:K], K)."""
+    _dev(keys, "keys")
+    idx = idx if idx is not None else torch.empty(T * N, dtype=torch.int32, device=keys.device)
+    K = _i32(0)
+    _check("echo_select_random", lib().echo_select_random(_p(keys), T, N, ratio_num, ratio_den,
+                                                          _p(idx), _c.byref(K), _stream(stream)))
+    return idx[:K.value], K.value
 
 
 def echo_step_delta_workspace_size(n: int) -> int:

@@ -163,3 +163,14 @@ def test_update_rate_rule_is_the_oracle_rule(ec):
         ec.echo_update_rate(float("nan"), 1.0, 100)
     with pytest.raises(ec.EchoError):
         ec.echo_update_rate(0.1, 1.0, 100, r_min=0.6, r_max=0.5)
+
+
+def test_ablation_selection_argument_checks(ec):
+    L = ec.lib()
+    K = ctypes.c_int32(-1)
+    assert L.echo_select_uniform(4, 64, 1, 4, None, ctypes.byref(K), None) == 1
+    assert L.echo_select_uniform(4, 64, 5, 4, _vp(FAKE), ctypes.byref(K), None) == 2
+    assert L.echo_select_uniform(0, 64, 1, 4, _vp(FAKE), ctypes.byref(K), None) == 2
+    assert L.echo_select_random(_vp(FAKE + 4), 4, 64, 1, 4, _vp(FAKE), ctypes.byref(K), None) == 1
+    assert L.echo_select_random(_vp(FAKE), 4, 64, 1, 0, _vp(FAKE), ctypes.byref(K), None) == 2
+    assert K.value == -1

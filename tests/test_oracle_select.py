@@ -137,3 +137,38 @@ def test_ratio_one_selects_all_ratio_zero_none():
     e = G.random_energy(3, seed=6)
     assert list(S.select(x, q, s, e, 3, 10, 1, 1)[0]) == list(range(30))
     assert len(S.select(x, q, s, e, 3, 10, 0, 1)[0]) == 0
+
+
+# ---- ablation selections (Sec. 4, Table 2: Uniform, Random) ----------------
+@pytest.mark.parametrize("NT,K", [(256, 64), (32760, 6552), (7, 3), (10, 10), (10, 1), (5, 0)])
+def test_uniform_selection_spacing(NT, K):
+    idx = S.uniform(NT, K)
+    assert len(idx) == K and idx.dtype == np.int32
+    if K:
+        assert idx[0] == 0 and np.all(np.diff(idx) > 0) and idx[-1] < NT
+        gaps = np.diff(np.append(idx, NT))
+        assert set(gaps.tolist()) <= {NT // K, -(-NT // K)}
+        # every window of ceil(NT/K) consecutive tokens holds at least one selected token
+        w = -(-NT // K)
+        hit = np.zeros(NT + w, dtype=int)
+        hit[idx] = 1
+        assert min(hit[i:i + w].sum() for i in range(NT - w + 1)) >= 1
+
+
+def test_random_subset_is_top_keys_and_uniform_in_frequency():
+    g = np.random.default_rng(0)
+    keys = g.random(12).astype(np.float32)
+    K = 5
+    # brute force: the subset of size K with the largest key sum is the top K
+    import itertools
+    best = max(itertools.combinations(range(12), K), key=lambda c: keys[list(c)].sum())
+    assert S.random_subset(keys, K).tolist() == sorted(best)
+    # equal keys: the lowest indices
+    assert S.random_subset(np.zeros(9, dtype=np.float32), 4).tolist() == [0, 1, 2, 3]
+    # with fresh uniform keys every token is picked with frequency K / NT
+    NT, trials = 40, 4000
+    cnt = np.zeros(NT)
+    for _ in range(trials):
+        cnt[S.random_subset(g.random(NT).astype(np.float32), 10)] += 1
+    f = cnt / trials
+    assert np.abs(f - 10 / NT).max() < 0.04
