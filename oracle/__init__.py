@@ -17,7 +17,9 @@ Modules:
             active) and the mask fusion.
   step    - one cached layer step, the step loop, the uncached block.
   schedule - step-level Eq. 1 change and the adaptive update rate r_t.
+  refcache - cache forms: plain int8, full precision (ablation), and the
+            reference-plus-int8-residual manager of Sec. 3.4.
 
 Parity status per function is stated in each module header.
 """
-from . import block, cache, energy, schedule, select, step  # noqa: F401
+from . import block, cache, energy, refcache, schedule, select, step  # noqa: F401

@@ -80,8 +80,13 @@ def dequant_f32(q: np.ndarray, s: np.ndarray) -> np.ndarray:
 
 def drift(x: np.ndarray, q: np.ndarray, s: np.ndarray, xi: float = 1e-6) -> np.ndarray:
     """d_i of Eq. 1 per token, fp32 [NT]."""
+    return drift_from(x, dequant_f32(q, s), xi)
+
+
+def drift_from(x: np.ndarray, c: np.ndarray, xi: float = 1e-6) -> np.ndarray:
+    """d_i of Eq. 1 against an fp32 reconstruction c of any cache form."""
     x = np.asarray(x, dtype=np.float32)
-    c = dequant_f32(q, s)
+    c = np.asarray(c, dtype=np.float32)
     num = canonical_sum(np.abs((x - c).astype(np.float32)))
     den = canonical_sum(np.abs(c))
     return (num / (den + np.float32(xi)).astype(np.float32)).astype(np.float32)
@@ -97,16 +102,23 @@ def refresh_budget(NT: int, ratio_num: int, ratio_den: int) -> int:
 def scores(x, q, s, seg_energy, T: int, N: int, lam: float = 0.1, xi: float = 1e-6,
            mode: int = MODE_ENERGY_DRIFT) -> np.ndarray:
     """score_i = w_{floor(i/N)} * d_i in fp32."""
+    return scores_from(x, None if mode == MODE_SEGMENT else dequant_f32(q, s), seg_energy, T, N,
+                       lam, xi, mode)
+
+
+def scores_from(x, c, seg_energy, T: int, N: int, lam: float = 0.1, xi: float = 1e-6,
+                mode: int = MODE_ENERGY_DRIFT) -> np.ndarray:
+    """scores against an fp32 reconstruction c of any cache form."""
     NT = T * N
     if mode == MODE_SEGMENT:
         w = segment_weights(seg_energy, 0.0)
         d = np.ones(NT, dtype=np.float32)
     elif mode == MODE_DRIFT_ONLY:
         w = np.ones(T, dtype=np.float32)
-        d = drift(x, q, s, xi)
+        d = drift_from(x, c, xi)
     else:
         w = segment_weights(seg_energy, lam)
-        d = drift(x, q, s, xi)
+        d = drift_from(x, c, xi)
     wt = np.repeat(w, N)
     return (wt * d).astype(np.float32)
 

@@ -62,6 +62,49 @@ def cached_layer_step(x, q, s, seg_energy, W, cond, T, N, H, ratio_num, ratio_de
     return LayerResult(idx, sc, y_act, y, y_bf16, q2, s2, bad)
 
 
+@dataclass
+class CacheLayerResult:
+    idx: np.ndarray          # int32 [K] ascending
+    scores: np.ndarray       # fp32 [NT] (zeros on a full step)
+    y_act: np.ndarray        # fp64 [K, D]
+    y: np.ndarray            # fp64 [NT, D], merged output
+    y_bf16: np.ndarray       # fp32 storage of bf16(y)
+    cache: object            # the cache after the write (a copy)
+    nonfinite: bool
+
+
+def cached_layer_step_cache(x, c, seg_energy, W, cond, T, N, H, ratio_num, ratio_den,
+                            lam=0.1, xi=1e-6, mode=select.MODE_ENERGY_DRIFT, full=False,
+                            idx=None) -> CacheLayerResult:
+    """The cached layer step with any cache form of refcache.py (Int8Cache,
+    FullCache, RefCache): the drift is taken against the form's fp32
+    reconstruction, inactive rows take its bf16 reconstruction, and the
+    refreshed rows are written through the form's own write.  The input cache
+    `c` is not modified."""
+    NT = T * N
+    if idx is not None:
+        idx = np.asarray(idx, dtype=np.int32)
+        sc = np.zeros(NT, dtype=np.float32)
+    elif full:
+        idx = np.arange(NT, dtype=np.int32)
+        sc = np.zeros(NT, dtype=np.float32)
+    else:
+        rec = None if mode == select.MODE_SEGMENT else c.reconstruct_f32()
+        sc = select.scores_from(x, rec, seg_energy, T, N, lam, xi, mode)
+        idx = select.top_k(sc, select.refresh_budget(NT, ratio_num, ratio_den))
+    cached = c.reconstruct_bf16()
+    if len(idx):
+        y_act = block.block_active(x, idx, W, cond, H)
+    else:
+        y_act = np.zeros((0, x.shape[1]))
+    y = block.merge(y_act, idx, cached)
+    c2 = c.copy()
+    bad = False
+    if len(idx):
+        bad = c2.write(idx, cache.round_bf16(y_act.astype(np.float32)))
+    return CacheLayerResult(idx, sc, y_act, y, cache.round_bf16(y.astype(np.float32)), c2, bad)
+
+
 def generation(x_inputs, weights, cond, seg_energy, T, N, H, ratio_num, ratio_den,
                lam=0.1, xi=1e-6, mode=select.MODE_ENERGY_DRIFT, warmup_steps=1,
                record=None, rate=None):

@@ -39,3 +39,14 @@ def test_hann_cosine_at_bin():
     n = np.arange(N)
     P = E.dft_power((np.cos(2 * np.pi * k0 * n / N) * E.hann_periodic(N))[None], N)[0]
     assert abs(P[k0] - g["P_k0"]) < 1e-9 and abs(P[k0 + 1] - g["P_neighbour"]) < 1e-9
+
+
+def test_ref_cache_scan():
+    from oracle import refcache as R
+    g = GOLD["ref_cache_scan"]
+    v = np.array(g["rows"], dtype=np.float32)
+    c = R.RefCache(len(v), v.shape[1], g["R_cap"], g["seg_len"], g["tau"])
+    rows = np.arange(len(v))
+    assert c.scan(rows, v).tolist() == g["src"]
+    c.write(rows, v)
+    assert c.ref.tolist() == g["ref"] and c.refcount.tolist() == g["refcount"]
