@@ -184,6 +184,105 @@ echo_status echo_select_static(const void *x, echo_dtype xt, const int8_t *cache
                                int32_t ratio_den, const echo_select_params *p,
                                int32_t *idx, int32_t *K_out, echo_stream_t stream);
 
+/* ---- cache forms (Sec. 3.4 and the quantisation ablation of Sec. 4, Table 2) ----
+ *
+ * One layer's cache of NT token rows of D values in one of three forms:
+ *   ECHO_CACHE_INT8  plain int8 per token ("Naive INT8"): c = bf16(float(q) s),
+ *                    the form echo_select / echo_block_step use.
+ *   ECHO_CACHE_BF16  the rows kept in the compute precision (the "FP16"
+ *                    ablation; compute precision here is bf16): c = full row.
+ *   ECHO_CACHE_REF   the paper's manager (Sec. 3.4): a row written to the cache
+ *                    is stored either as a reference (in full precision, in a
+ *                    pool slot) or as an int8 residual against the current
+ *                    reference: c = bf16(r + float(q) s), r = pool[ref] (0 when
+ *                    ref = -1).  Writing rows (ascending token order):
+ *                    1. release: every row about to be written drops its
+ *                       reference; a slot that no token refers to is free;
+ *                    2. scan: within each scan segment of seg_len consecutive
+ *                       tokens (segment floor(i / seg_len)) the first written
+ *                       row becomes the reference; a later row becomes the new
+ *                       reference when sim(x, r) <= tau, else it is stored as
+ *                       the int8 residual x - r.  sim = <x,r> / (sqrt(<x,x>)
+ *                       sqrt(<r,r>)) in fp32, the sums in the canonical order of
+ *                       the drift score, 0 when a norm is 0;
+ *                    3. allocation: new references in ascending token order
+ *                       take the free slots in ascending slot order; a
+ *                       reference that finds no free slot is not created and
+ *                       its whole run is stored as plain int8 (ref = -1);
+ *                    4. store: a reference copies its row into its slot with
+ *                       q = 0, s = 0; a residual is quantised by the int8 rule
+ *                       of echo_cache_quant; refcount[slot] counts the tokens
+ *                       whose entry names the slot.
+ *                    The paper gives neither tau, the scan order nor the pool
+ *                    size; seg_len = W' makes a segment one spatial row of a
+ *                    latent frame ("adjacent latents").
+ * All buffers are device memory owned by the caller, 16-byte aligned. */
+typedef enum { ECHO_CACHE_INT8 = 0, ECHO_CACHE_BF16 = 1, ECHO_CACHE_REF = 2 } echo_cache_kind;
+
+typedef struct {
+    int32_t kind;       /* echo_cache_kind */
+    int32_t NT;         /* tokens */
+    int32_t D;          /* values per token, multiple of 16 */
+    int8_t *q;          /* INT8, REF: int8 [NT, D] codes (REF: of the residual) */
+    float *scale;       /* INT8, REF: f32 [NT] */
+    void *full;         /* BF16: bf16 [NT, D] */
+    int32_t *ref;       /* REF: int32 [NT] pool slot of each token's reference, -1 = none */
+    void *pool;         /* REF: bf16 [R_cap, D] reference rows */
+    int32_t *refcount;  /* REF: int32 [R_cap], 0 = free slot */
+    int32_t R_cap;      /* REF: pool slots, >= 0 (0: every row plain int8) */
+    int32_t seg_len;    /* REF: tokens per scan segment, >= 1 */
+    float tau;          /* REF: similarity threshold */
+} echo_cache;
+
+/* Sets every entry of c to the empty state (q = 0, scale = 0, full = 0,
+ * ref = -1, refcount = 0): every token then reconstructs to 0.
+ * Errors: INVALID_ARG (descriptor), CUDA. */
+echo_status echo_cache_reset(const echo_cache *c, echo_stream_t stream);
+
+/* Bytes of device workspace echo_cache_write needs for n_rows rows (0 for
+ * INT8 and BF16). */
+size_t echo_cache_write_workspace_size(const echo_cache *c, int32_t n_rows);
+
+/* Writes src (bf16 [n_rows, D], device) into the cache at rows (int32
+ * [n_rows], device, ascending and distinct), by the rules of c's form.
+ * Errors: INVALID_ARG, SHAPE, WORKSPACE, CUDA; a non-finite row sets the
+ * NONFINITE device flag (INT8, REF: as echo_cache_quant). */
+echo_status echo_cache_write(const echo_cache *c, const void *src, const int32_t *rows,
+                             int32_t n_rows, void *workspace, size_t ws_bytes,
+                             echo_stream_t stream);
+
+/* dst[j] = the bf16 reconstruction c of token rows[j] (rows NULL: j), dst bf16
+ * [n_rows, D] device.  Errors: INVALID_ARG, SHAPE, CUDA. */
+echo_status echo_cache_read(const echo_cache *c, const int32_t *rows, int32_t n_rows, void *dst,
+                            echo_stream_t stream);
+
+/* REF only: out[0] = live references (slots with refcount > 0), out[1] = 1 +
+ * the highest live slot (the pool rows a caller needs to keep); out int32[2]
+ * device.  Errors: INVALID_ARG, CUDA. */
+echo_status echo_cache_stats(const echo_cache *c, int32_t *out, echo_stream_t stream);
+
+/* echo_select with the drift taken against the fp32 reconstruction of any
+ * cache form: INT8 float(q) s, BF16 the row, REF r + float(q) s (no bf16
+ * rounding).  Every other argument as echo_select. */
+echo_status echo_select_cache(const void *x, echo_dtype xt, const echo_cache *c,
+                              const float *seg_energy, int32_t T, int32_t N, int32_t ratio_num,
+                              int32_t ratio_den, const echo_select_params *p, int32_t *idx,
+                              int32_t *K_out, float *scores, void *workspace, size_t ws_bytes,
+                              echo_stream_t stream);
+
+/* Workspace of echo_block_step_cache: echo_workspace_size(dims, K_max) plus
+ * the cache write's. */
+size_t echo_block_step_cache_workspace_size(const echo_block_dims *dims, int32_t K_max,
+                                            const echo_cache *c);
+
+/* echo_block_step with any cache form: inactive rows take the bf16
+ * reconstruction of the cache as it was on entry, and the active rows are
+ * written with echo_cache_write's rules.  c->NT = T N and c->D = D. */
+echo_status echo_block_step_cache(const echo_block_weights *w, const echo_block_dims *dims,
+                                  const void *x, const int32_t *idx, int32_t K,
+                                  const echo_cache *c, void *y, void *workspace, size_t ws_bytes,
+                                  echo_stream_t stream);
+
 /* ---- ablation selections (Sec. 4, Table 2: "Uniform" and "Random" in place
  *      of the energy-guided anchor selection); no energy and no drift ---- */
 
@@ -331,7 +430,8 @@ typedef enum {
     ECHO_K_ENERGY = 0, ECHO_K_DRIFT = 1, ECHO_K_TOPK = 2, ECHO_K_ROWMAP = 3,
     ECHO_K_LAYERNORM = 4, ECHO_K_GEMM = 5, ECHO_K_ATTENTION = 6, ECHO_K_QUANT = 7,
     ECHO_K_DEQUANT = 8, ECHO_K_MERGE = 9, ECHO_K_STEP_DELTA = 10, ECHO_K_UNIFORM = 11,
-    ECHO_K_COUNT = 12
+    ECHO_K_REF_SCAN = 12, ECHO_K_REF_ALLOC = 13, ECHO_K_REF_STORE = 14, ECHO_K_CACHE_COPY = 15,
+    ECHO_K_COUNT = 16
 } echo_kernel_kind;
 
 /* Number of kernels this library has launched in this process (all devices). */
@@ -348,7 +448,8 @@ echo_status echo_profile_enable(int32_t on);
  * -1 on a CUDA error).  Shapes: GEMM (M, N, Kd); ATTENTION (M queries, L keys,
  * H * d); DRIFT (NT, D, 0); TOPK (NT, K, 0); LAYERNORM, QUANT, DEQUANT,
  * MERGE (rows, D, 0); ENERGY (T, frames, n_fft); STEP_DELTA (n, element bytes, 0)
- * for the reduction and (0, 0, blocks) for its final combine; UNIFORM (NT, K, 0). */
+ * for the reduction and (0, 0, blocks) for its final combine; UNIFORM (NT, K, 0);
+ * REF_SCAN, REF_ALLOC, REF_STORE, CACHE_COPY (rows, D, 0). */
 int32_t echo_profile_read(int32_t max, int32_t *kinds, int64_t *m, int64_t *n, int64_t *k,
                           float *ms);
 

@@ -170,7 +170,8 @@ extern "C" const char *echo_kernel_name(int32_t kind) {
     static const char *names[ECHO_K_COUNT] = {
         "segment_energy_fft", "drift_score",  "topk_select",  "rowmap",
         "layernorm_gather",   "gemm_tcgen05", "attention",    "quant_scatter",
-        "dequant_gather",     "dequant_merge", "step_delta",   "uniform_select"};
+        "dequant_gather",     "dequant_merge", "step_delta",   "uniform_select",
+        "ref_scan",           "ref_alloc",     "ref_store",    "cache_copy"};
     if (kind < 0 || kind >= ECHO_K_COUNT) return "unknown";
     return names[kind];
 }

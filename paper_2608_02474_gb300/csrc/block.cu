@@ -69,30 +69,33 @@ extern "C" echo_status echo_precompute_cross_kv(const void *cond, const void *Wk
                        2 * (int64_t)D, ECHO_BF16, stream);
 }
 
-extern "C" echo_status echo_block_step(const echo_block_weights *w, const echo_block_dims *dims,
-                                       const void *x, const int32_t *idx, int32_t K,
-                                       int8_t *cache_q, float *cache_scale, void *y,
-                                       void *workspace, size_t ws_bytes, echo_stream_t stream) {
+namespace {
+
+// argument checks shared by echo_block_step and echo_block_step_cache
+echo_status check_block(const echo_block_weights *w, const echo_block_dims *dims, const void *x,
+                        const int32_t *idx, int32_t K, const void *y, const void *workspace) {
     using namespace echo;
-    if (!w || !dims || !x || !cache_q || !cache_scale || !y || !workspace) return ECHO_ERR_INVALID_ARG;
+    if (!w || !dims || !x || !y || !workspace) return ECHO_ERR_INVALID_ARG;
     if (!dims_ok(dims)) return ECHO_ERR_SHAPE;
-    const echo_block_dims d = *dims;
-    const int NT = d.T * d.N;
+    const int NT = dims->T * dims->N;
     if (K < 0 || K > NT) return ECHO_ERR_SHAPE;
     if (K > 0 && !idx) return ECHO_ERR_INVALID_ARG;
     const void *ptrs[] = {w->Wq, w->bq, w->Wkv, w->bkv, w->Wo, w->bo, w->Wqc, w->bqc,
                           w->Woc, w->boc, w->W1, w->b1, w->W2, w->b2, w->KVc};
     for (const void *p : ptrs)
         if (!p || !aligned16(p)) return ECHO_ERR_INVALID_ARG;
-    if (!aligned16(x) || !aligned16(cache_q) || !aligned16(cache_scale) || !aligned16(y) ||
-        (idx && !aligned16(idx)) || (reinterpret_cast<uintptr_t>(workspace) & 255u))
+    if (!aligned16(x) || !aligned16(y) || (idx && !aligned16(idx)) ||
+        (reinterpret_cast<uintptr_t>(workspace) & 255u))
         return ECHO_ERR_INVALID_ARG;
-    const Layout L = layout(d, K);
-    if (ws_bytes < L.total) return ECHO_ERR_WORKSPACE;
-    if (!device_supported()) return ECHO_ERR_UNSUPPORTED;
+    return ECHO_OK;
+}
 
-    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    uint8_t *ws = static_cast<uint8_t *>(workspace);
+// rowmap and the block on the K active rows: y_act (bf16 [K, D]) at ws + L.yact
+echo_status run_active(const echo_block_weights *w, const echo_block_dims &d, const void *x,
+                       const int32_t *idx, int32_t K, uint8_t *ws, const Layout &L,
+                       cudaStream_t st) {
+    using namespace echo;
+    const int NT = d.T * d.N;
     int32_t *rowmap = reinterpret_cast<int32_t *>(ws + L.rowmap);
     void *n1 = ws + L.n1, *kv = ws + L.kv, *na = ws + L.na, *qa = ws + L.qa, *att = ws + L.att;
     void *h1 = ws + L.h1, *h2 = ws + L.h2, *u = ws + L.u, *yact = ws + L.yact;
@@ -100,7 +103,6 @@ extern "C" echo_status echo_block_step(const echo_block_weights *w, const echo_b
     const __nv_bfloat16 *kvb = static_cast<const __nv_bfloat16 *>(kv);
     const __nv_bfloat16 *kvc = static_cast<const __nv_bfloat16 *>(w->KVc);
     echo_status s = ECHO_OK;
-
     launch_rowmap(idx, K, NT, rowmap, st);
     if (K > 0) {
         launch_layernorm(x, ECHO_BF16, nullptr, NT, D, n1, st);
@@ -132,9 +134,69 @@ extern "C" echo_status echo_block_step(const echo_block_weights *w, const echo_b
                            ECHO_BF16}, st);
         if (s != ECHO_OK) return s;
     }
+    return last_launch_status();
+}
+
+}  // namespace
+
+extern "C" echo_status echo_block_step(const echo_block_weights *w, const echo_block_dims *dims,
+                                       const void *x, const int32_t *idx, int32_t K,
+                                       int8_t *cache_q, float *cache_scale, void *y,
+                                       void *workspace, size_t ws_bytes, echo_stream_t stream) {
+    using namespace echo;
+    echo_status s = check_block(w, dims, x, idx, K, y, workspace);
+    if (s != ECHO_OK) return s;
+    if (!cache_q || !cache_scale) return ECHO_ERR_INVALID_ARG;
+    if (!aligned16(cache_q) || !aligned16(cache_scale)) return ECHO_ERR_INVALID_ARG;
+    const echo_block_dims d = *dims;
+    const int NT = d.T * d.N;
+    const Layout L = layout(d, K);
+    if (ws_bytes < L.total) return ECHO_ERR_WORKSPACE;
+    if (!device_supported()) return ECHO_ERR_UNSUPPORTED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    s = run_active(w, d, x, idx, K, ws, L, st);
+    if (s != ECHO_OK) return s;
+    const int32_t *rowmap = reinterpret_cast<const int32_t *>(ws + L.rowmap);
     // the merge reads the cache of the inactive rows only, the quantiser writes
     // the active rows only: their order does not matter
-    launch_dequant_merge(cache_q, cache_scale, rowmap, yact, NT, D, y, st);
-    if (K > 0) launch_quant(yact, ECHO_BF16, idx, K, D, cache_q, cache_scale, st);
+    launch_dequant_merge(cache_q, cache_scale, rowmap, ws + L.yact, NT, d.D, y, st);
+    if (K > 0) launch_quant(ws + L.yact, ECHO_BF16, idx, K, d.D, cache_q, cache_scale, st);
     return last_launch_status();
+}
+
+extern "C" size_t echo_block_step_cache_workspace_size(const echo_block_dims *dims, int32_t K_max,
+                                                       const echo_cache *c) {
+    if (!dims_ok(dims) || K_max < 0 || echo::cache_check(c) != ECHO_OK) return 0;
+    return layout(*dims, K_max).total + echo::cache_write_ws(*c, K_max);
+}
+
+extern "C" echo_status echo_block_step_cache(const echo_block_weights *w,
+                                             const echo_block_dims *dims, const void *x,
+                                             const int32_t *idx, int32_t K, const echo_cache *c,
+                                             void *y, void *workspace, size_t ws_bytes,
+                                             echo_stream_t stream) {
+    using namespace echo;
+    echo_status s = check_block(w, dims, x, idx, K, y, workspace);
+    if (s != ECHO_OK) return s;
+    s = cache_check(c);
+    if (s != ECHO_OK) return s;
+    const echo_block_dims d = *dims;
+    if (c->NT != d.T * d.N || c->D != d.D) return ECHO_ERR_SHAPE;
+    const Layout L = layout(d, K);
+    const size_t wbytes = cache_write_ws(*c, K);
+    if (ws_bytes < L.total + wbytes) return ECHO_ERR_WORKSPACE;
+    if (!device_supported()) return ECHO_ERR_UNSUPPORTED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    s = run_active(w, d, x, idx, K, ws, L, st);
+    if (s != ECHO_OK) return s;
+    const int32_t *rowmap = reinterpret_cast<const int32_t *>(ws + L.rowmap);
+    // the merge reads the cache as it was on entry (the inactive rows and the
+    // references they name, which the write neither releases nor reuses);
+    // then the active rows are written
+    launch_cache_merge(*c, rowmap, ws + L.yact, y, st);
+    if (last_launch_status() != ECHO_OK) return ECHO_ERR_CUDA;
+    if (K > 0) return launch_cache_write(*c, ws + L.yact, idx, K, ws + L.total, st);
+    return ECHO_OK;
 }

@@ -67,4 +67,12 @@ void launch_rowmap(const int32_t *idx, int32_t K, int32_t NT, int32_t *rowmap, c
 void launch_dequant_merge(const int8_t *q, const float *scale, const int32_t *rowmap,
                           const void *y_act, int32_t NT, int32_t D, void *y, cudaStream_t st);
 
+// refcache.cu: cache forms other than plain int8 (and int8 through the same calls)
+echo_status cache_check(const echo_cache *c);
+size_t cache_write_ws(const echo_cache &c, int32_t n);
+echo_status launch_cache_write(const echo_cache &c, const void *src, const int32_t *rows,
+                               int32_t n, void *ws, cudaStream_t st);
+void launch_cache_merge(const echo_cache &c, const int32_t *rowmap, const void *y_act, void *y,
+                        cudaStream_t st);
+
 }  // namespace echo

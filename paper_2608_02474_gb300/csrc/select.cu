@@ -50,11 +50,24 @@ struct XChunk<float> {
     }
 };
 
-template <typename XT>
+// Where the drift reads the cached feature c_i from (Sec. 3.4 forms):
+//   kCacheInt8  c = float(q) * s
+//   kCacheBf16  c = the stored bf16 row (full-precision ablation)
+//   kCacheRef   c = r + float(q) * s, r the token's reference row (0 if none)
+struct CacheView {
+    const int8_t *q;
+    const float *scale;
+    const __nv_bfloat16 *full;
+    const int32_t *ref;
+    const __nv_bfloat16 *pool;
+};
+constexpr int kCacheInt8 = 0, kCacheBf16 = 1, kCacheRef = 2;
+
+template <typename XT, int CK>
 __global__ void __launch_bounds__(kDriftThreads)
-drift_kernel(const XT *__restrict__ x, const int8_t *__restrict__ q, const float *__restrict__ scale,
-             const float *__restrict__ seg_energy, int T, int N, int NT, int D, float lam, float xi,
-             int mode, float *__restrict__ scores, int *err) {
+drift_kernel(const XT *__restrict__ x, CacheView cv, const float *__restrict__ seg_energy, int T,
+             int N, int NT, int D, float lam, float xi, int mode, float *__restrict__ scores,
+             int *err) {
     __shared__ float s_emax;
     if (threadIdx.x < 32) {
         float m = 0.f;
@@ -78,32 +91,47 @@ drift_kernel(const XT *__restrict__ x, const int8_t *__restrict__ q, const float
 
         float d = 1.f;
         if (mode != ECHO_MODE_SEGMENT) {
-            const float sc = scale[row];
+            const float sc = CK == kCacheBf16 ? 0.f : cv.scale[row];
             const XT *xr = x + (int64_t)row * D;
-            const int8_t *qr = q + (int64_t)row * D;
+            const int8_t *qr = CK == kCacheBf16 ? nullptr : cv.q + (int64_t)row * D;
+            const __nv_bfloat16 *fr = nullptr;
+            if constexpr (CK == kCacheBf16) fr = cv.full + (int64_t)row * D;
+            if constexpr (CK == kCacheRef) {
+                const int rs = cv.ref[row];
+                fr = rs >= 0 ? cv.pool + (int64_t)rs * D : nullptr;
+            }
             float num = 0.f, den = 0.f;
             for (int c0 = lane; c0 < C; c0 += 32 * kDriftUnroll) {
                 XChunk<XT> xv[kDriftUnroll];
                 uint2 qv[kDriftUnroll];
+                uint4 fv[kDriftUnroll];
 #pragma unroll
                 for (int u = 0; u < kDriftUnroll; ++u) {
                     const int c = c0 + 32 * u;
                     if (c < C) {
                         xv[u].load(xr + 8 * c);
-                        qv[u] = __ldcs(reinterpret_cast<const uint2 *>(qr + 8 * c));
+                        if constexpr (CK != kCacheBf16)
+                            qv[u] = __ldcs(reinterpret_cast<const uint2 *>(qr + 8 * c));
+                        if constexpr (CK != kCacheInt8)
+                            fv[u] = fr ? __ldcs(reinterpret_cast<const uint4 *>(fr + 8 * c))
+                                       : make_uint4(0, 0, 0, 0);
                     }
                 }
 #pragma unroll
                 for (int u = 0; u < kDriftUnroll; ++u) {
                     const int c = c0 + 32 * u;
                     if (c < C) {
-                        float xf[8];
+                        float xf[8], rf[8];
                         xv[u].get(xf);
+                        if constexpr (CK != kCacheInt8) unpack8_bf16(fv[u], rf);
                         const int8_t *qb = reinterpret_cast<const int8_t *>(&qv[u]);
                         float cn = 0.f, cd = 0.f;
 #pragma unroll
                         for (int k = 0; k < 8; ++k) {
-                            const float ch = __fmul_rn((float)qb[k], sc);
+                            float ch;
+                            if constexpr (CK == kCacheInt8) ch = __fmul_rn((float)qb[k], sc);
+                            else if constexpr (CK == kCacheBf16) ch = rf[k];
+                            else ch = __fadd_rn(rf[k], __fmul_rn((float)qb[k], sc));
                             const float an = fabsf(__fsub_rn(xf[k], ch));
                             const float ad = fabsf(ch);
                             cn = k ? __fadd_rn(cn, an) : an;
@@ -318,13 +346,13 @@ extern "C" echo_status echo_select(const void *x, echo_dtype xt, const int8_t *c
     {
     LaunchScope ls(ECHO_K_DRIFT, NT, D, 0, st);
     if (xt == ECHO_BF16)
-        drift_kernel<__nv_bfloat16><<<grid, kDriftThreads, 0, st>>>(
-            static_cast<const __nv_bfloat16 *>(x), cache_q, cache_scale, seg_energy, T, N, NT, D,
-            prm.lambda, prm.xi, prm.mode, sc, err);
+        drift_kernel<__nv_bfloat16, kCacheInt8><<<grid, kDriftThreads, 0, st>>>(
+            static_cast<const __nv_bfloat16 *>(x), CacheView{cache_q, cache_scale, nullptr, nullptr,
+            nullptr}, seg_energy, T, N, NT, D, prm.lambda, prm.xi, prm.mode, sc, err);
     else
-        drift_kernel<float><<<grid, kDriftThreads, 0, st>>>(
-            static_cast<const float *>(x), cache_q, cache_scale, seg_energy, T, N, NT, D,
-            prm.lambda, prm.xi, prm.mode, sc, err);
+        drift_kernel<float, kCacheInt8><<<grid, kDriftThreads, 0, st>>>(
+            static_cast<const float *>(x), CacheView{cache_q, cache_scale, nullptr, nullptr,
+            nullptr}, seg_energy, T, N, NT, D, prm.lambda, prm.xi, prm.mode, sc, err);
     }
     if (last_launch_status() != ECHO_OK) return ECHO_ERR_CUDA;
 
@@ -410,13 +438,13 @@ extern "C" echo_status echo_select_static(const void *x, echo_dtype xt, const in
     {
         LaunchScope ls(ECHO_K_DRIFT, NT, D, 0, st);
         if (xt == ECHO_BF16)
-            drift_kernel<__nv_bfloat16><<<grid, kDriftThreads, 0, st>>>(
-                static_cast<const __nv_bfloat16 *>(x), cache_q, cache_scale, seg_energy, T, N, NT,
-                D, prm.lambda, prm.xi, prm.mode, sc, err);
+            drift_kernel<__nv_bfloat16, kCacheInt8><<<grid, kDriftThreads, 0, st>>>(
+                static_cast<const __nv_bfloat16 *>(x), CacheView{cache_q, cache_scale, nullptr,
+                nullptr, nullptr}, seg_energy, T, N, NT, D, prm.lambda, prm.xi, prm.mode, sc, err);
         else
-            drift_kernel<float><<<grid, kDriftThreads, 0, st>>>(
-                static_cast<const float *>(x), cache_q, cache_scale, seg_energy, T, N, NT, D,
-                prm.lambda, prm.xi, prm.mode, sc, err);
+            drift_kernel<float, kCacheInt8><<<grid, kDriftThreads, 0, st>>>(
+                static_cast<const float *>(x), CacheView{cache_q, cache_scale, nullptr, nullptr,
+                nullptr}, seg_energy, T, N, NT, D, prm.lambda, prm.xi, prm.mode, sc, err);
     }
     if (last_launch_status() != ECHO_OK) return ECHO_ERR_CUDA;
     const size_t key_bytes = (size_t)NT * sizeof(uint32_t);
@@ -485,6 +513,82 @@ extern "C" echo_status echo_select_random(const float *keys, int32_t T, int32_t 
     {
         LaunchScope ls(ECHO_K_TOPK, NT, K, 0, st);
         topk_kernel<<<1, kTopkThreads, dyn, st>>>(keys, NT, K, in_smem, idx);
+    }
+    return last_launch_status();
+}
+
+extern "C" echo_status echo_select_cache(const void *x, echo_dtype xt, const echo_cache *c,
+                                         const float *seg_energy, int32_t T, int32_t N,
+                                         int32_t ratio_num, int32_t ratio_den,
+                                         const echo_select_params *p, int32_t *idx,
+                                         int32_t *K_out, float *scores, void *workspace,
+                                         size_t ws_bytes, echo_stream_t stream) {
+    using namespace echo;
+    const echo_status v = cache_check(c);
+    if (v != ECHO_OK) return v;
+    if (c->kind == ECHO_CACHE_INT8)
+        return echo_select(x, xt, c->q, c->scale, seg_energy, T, N, c->D, ratio_num, ratio_den, p,
+                           idx, K_out, scores, workspace, ws_bytes, stream);
+    if (!x || !seg_energy || !idx || !K_out) return ECHO_ERR_INVALID_ARG;
+    if (xt != ECHO_BF16 && xt != ECHO_F32) return ECHO_ERR_INVALID_ARG;
+    if (!aligned16(x) || !aligned16(seg_energy) || !aligned16(idx) || (scores && !aligned16(scores)))
+        return ECHO_ERR_INVALID_ARG;
+    echo_select_params prm = {0.1f, 1e-6f, ECHO_MODE_ENERGY_DRIFT};
+    if (p) prm = *p;
+    if (prm.mode < 0 || prm.mode > 2 || !(prm.xi > 0.f) || !(prm.lambda >= 0.f) ||
+        !(prm.lambda <= 1.f))
+        return ECHO_ERR_INVALID_ARG;
+    if (T < 1 || N < 1 || ratio_den < 1 || ratio_num < 0 || ratio_num > ratio_den)
+        return ECHO_ERR_SHAPE;
+    if ((int64_t)T * N != c->NT) return ECHO_ERR_SHAPE;
+    const int NT = c->NT, D = c->D;
+    const int K = (int)(((int64_t)ratio_num * NT + ratio_den - 1) / ratio_den);
+    float *sc = scores;
+    if (!sc) {
+        if (!workspace || !aligned16(workspace)) return ECHO_ERR_INVALID_ARG;
+        if (ws_bytes < echo_select_workspace_size(T, N)) return ECHO_ERR_WORKSPACE;
+        sc = static_cast<float *>(workspace);
+    }
+    if (!device_supported()) return ECHO_ERR_UNSUPPORTED;
+    *K_out = K;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    int *err = device_error_ptr();
+    const CacheView cv{c->q, c->scale, static_cast<const __nv_bfloat16 *>(c->full), c->ref,
+                       static_cast<const __nv_bfloat16 *>(c->pool)};
+    const int warps = kDriftThreads / 32;
+    const int grid = (NT + warps - 1) / warps;
+    {
+        LaunchScope ls(ECHO_K_DRIFT, NT, D, 0, st);
+        const bool bf = xt == ECHO_BF16;
+        const __nv_bfloat16 *xb = static_cast<const __nv_bfloat16 *>(x);
+        const float *xf = static_cast<const float *>(x);
+        if (c->kind == ECHO_CACHE_BF16) {
+            if (bf)
+                drift_kernel<__nv_bfloat16, kCacheBf16><<<grid, kDriftThreads, 0, st>>>(
+                    xb, cv, seg_energy, T, N, NT, D, prm.lambda, prm.xi, prm.mode, sc, err);
+            else
+                drift_kernel<float, kCacheBf16><<<grid, kDriftThreads, 0, st>>>(
+                    xf, cv, seg_energy, T, N, NT, D, prm.lambda, prm.xi, prm.mode, sc, err);
+        } else {
+            if (bf)
+                drift_kernel<__nv_bfloat16, kCacheRef><<<grid, kDriftThreads, 0, st>>>(
+                    xb, cv, seg_energy, T, N, NT, D, prm.lambda, prm.xi, prm.mode, sc, err);
+            else
+                drift_kernel<float, kCacheRef><<<grid, kDriftThreads, 0, st>>>(
+                    xf, cv, seg_energy, T, N, NT, D, prm.lambda, prm.xi, prm.mode, sc, err);
+        }
+    }
+    if (last_launch_status() != ECHO_OK) return ECHO_ERR_CUDA;
+    const size_t key_bytes = (size_t)NT * sizeof(uint32_t);
+    const int in_smem = key_bytes <= 200 * 1024 ? 1 : 0;
+    const size_t dyn = in_smem ? key_bytes : 0;
+    if (dyn > 48 * 1024 &&
+        cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn) !=
+            cudaSuccess)
+        return ECHO_ERR_CUDA;
+    {
+        LaunchScope ls(ECHO_K_TOPK, NT, K, 0, st);
+        topk_kernel<<<1, kTopkThreads, dyn, st>>>(sc, NT, K, in_smem, idx);
     }
     return last_launch_status();
 }

@@ -11,6 +11,7 @@ import ctypes
 import os
 from dataclasses import dataclass
 
+import numpy as np
 import torch
 
 HERE = os.path.dirname(os.path.abspath(__file__))
@@ -39,6 +40,15 @@ class RateParams(_c.Structure):
     _fields_ = [("r_min", _f64), ("r_max", _f64), ("alpha", _f64)]
 
 
+CACHE_INT8, CACHE_BF16, CACHE_REF = 0, 1, 2
+
+
+class CacheC(_c.Structure):
+    _fields_ = [("kind", _i32), ("NT", _i32), ("D", _i32), ("q", _vp), ("scale", _vp),
+                ("full", _vp), ("ref", _vp), ("pool", _vp), ("refcount", _vp), ("R_cap", _i32),
+                ("seg_len", _i32), ("tau", _f32)]
+
+
 class BlockDims(_c.Structure):
     _fields_ = [("T", _i32), ("N", _i32), ("D", _i32), ("H", _i32), ("d", _i32), ("F", _i32),
                 ("Lc", _i32)]
@@ -58,6 +68,18 @@ _SIGS = {
                            _c.POINTER(SelectParams), _vp, _c.POINTER(_i32), _vp, _vp, _sz, _vp]),
     "echo_select_static": (_i32, [_vp, _i32, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32,
                                   _c.POINTER(SelectParams), _vp, _c.POINTER(_i32), _vp]),
+    "echo_cache_reset": (_i32, [_c.POINTER(CacheC), _vp]),
+    "echo_cache_write_workspace_size": (_sz, [_c.POINTER(CacheC), _i32]),
+    "echo_cache_write": (_i32, [_c.POINTER(CacheC), _vp, _vp, _i32, _vp, _sz, _vp]),
+    "echo_cache_read": (_i32, [_c.POINTER(CacheC), _vp, _i32, _vp, _vp]),
+    "echo_cache_stats": (_i32, [_c.POINTER(CacheC), _vp, _vp]),
+    "echo_select_cache": (_i32, [_vp, _i32, _c.POINTER(CacheC), _vp, _i32, _i32, _i32, _i32,
+                                 _c.POINTER(SelectParams), _vp, _c.POINTER(_i32), _vp, _vp, _sz,
+                                 _vp]),
+    "echo_block_step_cache_workspace_size": (_sz, [_c.POINTER(BlockDims), _i32,
+                                                   _c.POINTER(CacheC)]),
+    "echo_block_step_cache": (_i32, [_c.POINTER(BlockWeightsC), _c.POINTER(BlockDims), _vp, _vp,
+                                     _i32, _c.POINTER(CacheC), _vp, _vp, _sz, _vp]),
     "echo_select_uniform": (_i32, [_i32, _i32, _i32, _i32, _vp, _c.POINTER(_i32), _vp]),
     "echo_select_random": (_i32, [_vp, _i32, _i32, _i32, _i32, _vp, _c.POINTER(_i32), _vp]),
     "echo_step_delta_workspace_size": (_sz, [_i64]),
@@ -349,3 +371,133 @@ class DeviceBlock:
         t["KVc"] = echo_precompute_cross_kv(bf(cond), Wkvc, bkvc, stream=stream)
         c = BlockWeightsC(*[_p(t[n]) for n, _ in BlockWeightsC._fields_])
         return DeviceBlock(t, c)
+
+
+class DeviceCache:
+    """One layer's cache in one of the forms of echo_cache, with its device
+    tensors owned here.  kind CACHE_INT8: q, scale; CACHE_BF16: full;
+    CACHE_REF: q, scale, ref, pool [R_cap, D], refcount (R_cap defaults to NT,
+    the most references a cache can hold; seg_len, tau as echo_cache).
+    Starts empty (echo_cache_reset)."""
+
+    def __init__(self, kind: int, NT: int, D: int, R_cap: int | None = None, seg_len: int = 1,
+                 tau: float = 0.9, device="cuda", stream=None):
+        dev = torch.device(device)
+        self.kind, self.NT, self.D = kind, NT, D
+        self.t = {}
+        if kind in (CACHE_INT8, CACHE_REF):
+            self.t["q"] = torch.empty(NT, D, dtype=torch.int8, device=dev)
+            self.t["scale"] = torch.empty(NT, dtype=torch.float32, device=dev)
+        if kind == CACHE_BF16:
+            self.t["full"] = torch.empty(NT, D, dtype=torch.bfloat16, device=dev)
+        R_cap = (NT if R_cap is None else R_cap) if kind == CACHE_REF else 0
+        if kind == CACHE_REF:
+            self.t["ref"] = torch.empty(NT, dtype=torch.int32, device=dev)
+            self.t["pool"] = torch.empty(max(R_cap, 1), D, dtype=torch.bfloat16, device=dev)
+            self.t["refcount"] = torch.empty(max(R_cap, 1), dtype=torch.int32, device=dev)
+        self.R_cap, self.seg_len, self.tau = R_cap, seg_len, tau
+        self.cstruct = CacheC(kind, NT, D, *[_p(self.t.get(n)) for n in
+                                             ("q", "scale", "full", "ref", "pool", "refcount")],
+                              R_cap, seg_len, tau)
+        self.reset(stream)
+
+    def reset(self, stream=None):
+        _check("echo_cache_reset", lib().echo_cache_reset(_c.byref(self.cstruct), _stream(stream)))
+
+    def load(self, **arrays):
+        """Overwrite state tensors (q, scale, full, ref, pool, refcount) from
+        host arrays of the same shapes (pool and full as bf16 values)."""
+        for n, a in arrays.items():
+            t = self.t[n]
+            src = torch.as_tensor(np.ascontiguousarray(a)).to(t.dtype)
+            t[:src.shape[0]].copy_(src.to(t.device))
+
+    def clone(self) -> "DeviceCache":
+        c = DeviceCache.__new__(DeviceCache)
+        c.kind, c.NT, c.D = self.kind, self.NT, self.D
+        c.R_cap, c.seg_len, c.tau = self.R_cap, self.seg_len, self.tau
+        c.t = {n: t.clone() for n, t in self.t.items()}
+        c.cstruct = CacheC(c.kind, c.NT, c.D, *[_p(c.t.get(n)) for n in
+                                               ("q", "scale", "full", "ref", "pool", "refcount")],
+                           c.R_cap, c.seg_len, c.tau)
+        return c
+
+    def write_workspace_size(self, n_rows: int) -> int:
+        return lib().echo_cache_write_workspace_size(_c.byref(self.cstruct), n_rows)
+
+    def write(self, src, rows, workspace=None, stream=None):
+        _dev(src, "src")
+        _dev(rows, "rows")
+        n = rows.numel()
+        need = self.write_workspace_size(n)
+        if workspace is None and need:
+            workspace = torch.empty(need, dtype=torch.uint8, device=src.device)
+        wsb = 0 if workspace is None else workspace.numel()
+        _check("echo_cache_write", lib().echo_cache_write(
+            _c.byref(self.cstruct), _p(src), _p(rows), n, _p(workspace), wsb, _stream(stream)))
+
+    def read(self, rows=None, out=None, stream=None):
+        n = self.NT if rows is None else rows.numel()
+        dev = self.t["q" if "q" in self.t else "full"].device
+        out = out if out is not None else torch.empty(n, self.D, dtype=torch.bfloat16, device=dev)
+        _check("echo_cache_read", lib().echo_cache_read(_c.byref(self.cstruct), _p(rows), n,
+                                                        _p(out), _stream(stream)))
+        return out
+
+    def stats(self, stream=None) -> tuple[int, int]:
+        """(live references, high-water mark); synchronises the stream."""
+        out = torch.zeros(2, dtype=torch.int32, device=self.t["ref"].device)
+        _check("echo_cache_stats", lib().echo_cache_stats(_c.byref(self.cstruct), _p(out),
+                                                          _stream(stream)))
+        a, b = out.cpu().tolist()
+        return a, b
+
+    def nbytes(self, pool_rows: int | None = None) -> int:
+        """Device bytes of this cache; for CACHE_REF with `pool_rows`, the bytes
+        of a pool sized to that many rows instead of R_cap."""
+        total = 0
+        for n, t in self.t.items():
+            if n in ("pool", "refcount") and pool_rows is not None:
+                total += pool_rows * t[0].numel() * t.element_size()
+            else:
+                total += t.numel() * t.element_size()
+        return total
+
+
+def echo_select_cache(x, cache: DeviceCache, seg_energy, T: int, N: int, ratio_num: int,
+                      ratio_den: int, lam: float = 0.1, xi: float = 1e-6,
+                      mode: int = MODE_ENERGY_DRIFT, idx=None, scores=None, workspace=None,
+                      stream=None):
+    """echo_select against any cache form; returns (idx[:K] int32, K, scores or None)."""
+    _dev(x, "x")
+    _dev(seg_energy, "seg_energy")
+    NT = x.shape[0]
+    idx = idx if idx is not None else torch.empty(NT, dtype=torch.int32, device=x.device)
+    if scores is None and workspace is None:
+        workspace = torch.empty(echo_select_workspace_size(T, N), dtype=torch.uint8, device=x.device)
+    prm = SelectParams(lam, xi, mode)
+    K = _i32(0)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check("echo_select_cache", lib().echo_select_cache(
+        _p(x), _dtype(x), _c.byref(cache.cstruct), _p(seg_energy), T, N, ratio_num, ratio_den,
+        _c.byref(prm), _p(idx), _c.byref(K), _p(scores), _p(workspace), ws_bytes,
+        _stream(stream)))
+    return idx[:K.value], K.value, scores
+
+
+def echo_block_step_cache_workspace_size(dims: BlockDims, K_max: int, cache: DeviceCache) -> int:
+    return lib().echo_block_step_cache_workspace_size(_c.byref(dims), K_max,
+                                                      _c.byref(cache.cstruct))
+
+
+def echo_block_step_cache(weights: DeviceBlock, dims: BlockDims, x, idx, K: int,
+                          cache: DeviceCache, y=None, workspace=None, stream=None):
+    y = y if y is not None else torch.empty_like(x)
+    if workspace is None:
+        workspace = torch.empty(echo_block_step_cache_workspace_size(dims, K, cache),
+                                dtype=torch.uint8, device=x.device)
+    _check("echo_block_step_cache", lib().echo_block_step_cache(
+        _c.byref(weights.cstruct), _c.byref(dims), _p(x), _p(idx) if K > 0 else None, K,
+        _c.byref(cache.cstruct), _p(y), _p(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
+    return y

@@ -157,3 +157,18 @@ def step_output_pair(n: int, seed: int, change: float = 0.05, bf16: bool = True)
     if bf16:
         return to_bf16_values(a), to_bf16_values(b)
     return a, b
+
+
+def correlated_rows(n: int, D: int, seed: int, rho: float = 0.95) -> np.ndarray:
+    """[n, D] bf16 values; consecutive rows follow an AR(1) chain,
+    x_i = rho x_{i-1} + sqrt(1 - rho^2) e_i with e ~ N(0, 1), so neighbouring
+    rows have cosine similarity about rho (like spatially adjacent latents)."""
+    g = rng(seed)
+    e = g.standard_normal((n, D), dtype=np.float32)
+    x = np.empty_like(e)
+    if n:
+        x[0] = e[0]
+    c = np.float32(np.sqrt(1.0 - rho * rho))
+    for i in range(1, n):
+        x[i] = np.float32(rho) * x[i - 1] + c * e[i]
+    return to_bf16_values(x)

@@ -174,3 +174,30 @@ def test_ablation_selection_argument_checks(ec):
     assert L.echo_select_random(_vp(FAKE + 4), 4, 64, 1, 4, _vp(FAKE), ctypes.byref(K), None) == 1
     assert L.echo_select_random(_vp(FAKE), 4, 64, 1, 0, _vp(FAKE), ctypes.byref(K), None) == 2
     assert K.value == -1
+
+
+def test_cache_form_argument_checks(ec):
+    L = ec.lib()
+    mk = lambda kind=2, NT=64, D=64, ref=FAKE, R_cap=64, seg=8: ec.CacheC(
+        kind, NT, D, FAKE, FAKE, FAKE, ref, FAKE, FAKE, R_cap, seg, 0.9)
+    c = mk()
+    assert ec.lib().echo_cache_write_workspace_size(ctypes.byref(c), 64) > 0
+    assert L.echo_cache_write(ctypes.byref(mk(kind=7)), _vp(FAKE), _vp(FAKE), 4, _vp(FAKE),
+                              1 << 20, None) == 1
+    assert L.echo_cache_write(ctypes.byref(mk(D=24)), _vp(FAKE), _vp(FAKE), 4, _vp(FAKE),
+                              1 << 20, None) == 2
+    assert L.echo_cache_write(ctypes.byref(mk(ref=0)), _vp(FAKE), _vp(FAKE), 4, _vp(FAKE),
+                              1 << 20, None) == 1
+    assert L.echo_cache_write(ctypes.byref(mk(seg=0)), _vp(FAKE), _vp(FAKE), 4, _vp(FAKE),
+                              1 << 20, None) == 1
+    assert L.echo_cache_write(ctypes.byref(c), _vp(FAKE), _vp(FAKE), 65, _vp(FAKE),
+                              1 << 20, None) == 2
+    assert L.echo_cache_write(ctypes.byref(c), _vp(FAKE), _vp(FAKE), 4, _vp(FAKE), 16, None) == 3
+    assert L.echo_cache_write(ctypes.byref(c), _vp(FAKE), _vp(FAKE), 0, None, 0, None) == 0
+    assert L.echo_cache_stats(ctypes.byref(mk(kind=1)), _vp(FAKE), None) == 1
+    dims = ec.BlockDims(4, 16, 64, 1, 64, 128, 8)
+    w = ec.BlockWeightsC(*([FAKE] * 15))
+    # the cache must match the block's NT and D
+    assert L.echo_block_step_cache(ctypes.byref(w), ctypes.byref(dims), _vp(FAKE), _vp(FAKE), 4,
+                                   ctypes.byref(mk(NT=65)), _vp(FAKE), _vp(FAKE), 1 << 30,
+                                   None) == 2
