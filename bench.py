@@ -48,6 +48,18 @@ def parse():
                     help="adaptive update rate (Sec. 3.3) instead of a fixed ratio, e.g. "
                          "0.1,0.5,0.2; the change of Eq. 1 between consecutive step outputs "
                          "and the host rule are part of every timed step")
+    ap.add_argument("--cache", default="int8", choices=["int8", "bf16", "ref"],
+                    help="cache form: plain int8 (default), full-precision bf16 (ablation) or "
+                         "reference plus int8 residual (Sec. 3.4)")
+    ap.add_argument("--tau", type=float, default=0.9, help="--cache ref: similarity threshold")
+    ap.add_argument("--seg-len", type=int, default=0,
+                    help="--cache ref: tokens per scan segment (default: the frame width W')")
+    ap.add_argument("--select", default="energy", choices=["energy", "uniform", "random"],
+                    help="token selection: energy-guided (default) or the Uniform / Random "
+                         "ablations")
+    ap.add_argument("--latents", default="iid", choices=["iid", "smooth"],
+                    help="synthetic latents: i.i.d. (default) or spatially smooth rows "
+                         "(AR(1) along each frame row, rho 0.95)")
     ap.add_argument("--sweep", action="store_true",
                     help="refresh-ratio x audio-profile sweep against the uncached block "
                          "(one JSON line per point and a break-even summary)")
@@ -201,25 +213,44 @@ def load_peaks():
 
 
 # ---------------------------------------------------------------------------
-def oracle_sample(w, audio, W, cond, x1, q, s, rnum, rden, budget_s=25.0, adaptive=False):
+def oracle_sample(w, audio, W, cond, x1, q, s, rnum, rden, budget_s=25.0, adaptive=False,
+                  form="int8", selection="energy", tau=0.9, seg_len=None):
     """Time the CPU oracle on a bounded sample of one cached step and extrapolate.
 
-    Measured in full: audio energy, drift + top-K over all tokens, the merge
-    (reconstruction of the inactive rows) and the int8 write of the active rows.
+    Measured in full: audio energy, drift + top-K over all tokens (or the
+    Uniform / Random selection), the merge (reconstruction of the inactive
+    rows) and the cache write of the active rows in the cache form asked for.
     Sampled: K/V projection of `s_kv` rows (scaled by NT / s_kv) and the
     active-row block (Q', attention over all NT keys, cross-attention, FFN) of
-    `s_a` rows (scaled by K / s_a)."""
+    `s_a` rows (scaled by K / s_a).  The cache starts as the cache form of the
+    previous step's rows q, s reconstruct to."""
     import numpy as np
     import oracle
     t = {}
+    prev = oracle.cache.dequantize_rows(q, s)
+    if form == "int8":
+        c = oracle.refcache.Int8Cache(w.NT, w.D)
+        c.q, c.s = q.copy(), s.copy()
+    elif form == "bf16":
+        c = oracle.refcache.FullCache(w.NT, w.D)
+        c.v = prev
+    else:
+        c = oracle.refcache.RefCache(w.NT, w.D, w.NT, seg_len or w.Wp, tau)
+        c.write(np.arange(w.NT), prev)
     t0 = time.perf_counter()
     _, e = oracle.energy.audio_energy(audio, w.T)
     t["energy"] = time.perf_counter() - t0
     e32 = e.astype(np.float32)
     t0 = time.perf_counter()
-    idx, _ = oracle.select.select(x1, q, s, e32, w.T, w.N, rnum, rden)
+    K = oracle.select.refresh_budget(w.NT, rnum, rden)
+    if selection == "uniform":
+        idx = oracle.select.uniform(w.NT, K)
+    elif selection == "random":
+        idx = oracle.select.random_subset(np.random.default_rng(0).random(w.NT, dtype=np.float32), K)
+    else:
+        sc = oracle.select.scores_from(x1, c.reconstruct_f32(), e32, w.T, w.N)
+        idx = oracle.select.top_k(sc, K)
     t["select"] = time.perf_counter() - t0
-    K = len(idx)
     s_kv = min(w.NT, 4096)
     t0 = time.perf_counter()
     oracle.block.self_kv(x1[:s_kv], W)
@@ -230,24 +261,23 @@ def oracle_sample(w, audio, W, cond, x1, q, s, rnum, rden, budget_s=25.0, adapti
     t0 = time.perf_counter()
     oracle.block.active_rows(x1, idx[:s_a], W, w.H, kv_stand_in, kv_stand_in, Kc, Vc)
     t["active_sample"] = time.perf_counter() - t0
-    inactive = np.setdiff1d(np.arange(w.NT), idx)
     t0 = time.perf_counter()
-    oracle.cache.dequantize_rows(q[inactive], s[inactive])
-    qq, ss = q.copy(), s.copy()
-    oracle.cache.quant_scatter(x1[idx], idx, qq, ss)
-    t["merge_quant"] = time.perf_counter() - t0
+    c.reconstruct_bf16()
+    c.write(idx, x1[idx])
+    t["merge_write"] = time.perf_counter() - t0
     per_layer = (t["select"] + t["kv_sample"] * w.NT / s_kv + t["active_sample"] * K / s_a
-                 + t["merge_quant"])
+                 + t["merge_write"])
     step_s = t["energy"] + w.layers * per_layer
     if adaptive:
         t0 = time.perf_counter()
         oracle.schedule.step_delta(kv_stand_in, x1)   # two [NT, D] arrays: timing only
         t["step_delta"] = time.perf_counter() - t0
         step_s += t["step_delta"]
-    sample = (f"oracle on one {w.name} cached step: energy, drift+top-K over all {w.NT} tokens, "
-              f"merge and int8 write in full; K/V projection timed on {s_kv} of {w.NT} rows and "
-              f"the active-row block on {s_a} of {K} rows, each scaled to the full count; "
-              f"one layer timed, times {w.layers} layers"
+    sel = "drift+top-K over all" if selection == "energy" else f"{selection} selection of"
+    sample = (f"oracle on one {w.name} cached step: energy, {sel} {w.NT} tokens, "
+              f"merge and {form} cache write in full; K/V projection timed on {s_kv} of {w.NT} "
+              f"rows and the active-row block on {s_a} of {K} rows, each scaled to the full "
+              f"count; one layer timed, times {w.layers} layers"
               + ("; the step-level Eq. 1 change over all NT x D values in full" if adaptive else "")
               + f"; {sum(t.values()):.1f} s of CPU time")
     return step_s, sample, t
@@ -261,13 +291,13 @@ def cpu_cores():
 
 
 # ---------------------------------------------------------------------------
-def build_inputs(w, profile):
+def build_inputs(w, profile, latents="iid"):
     import numpy as np
     from synth import generate as G
     audio = G.audio(w, profile)
     W = G.block_weights(w, 0)
     cond = G.cond_tokens(w, audio)
-    x0 = G.latents(w)
+    x0 = G.latents(w) if latents == "iid" else G.latents_smooth(w)
     xs = [G.step_input(w, x0, t) for t in (1, 2)]
     return audio, W, cond, x0, xs
 
@@ -277,11 +307,13 @@ def run_reference(args, w, rnum, rden, rank):
         return
     import numpy as np
     import oracle
-    audio, W, cond, x0, xs = build_inputs(w, args.profile)
+    audio, W, cond, x0, xs = build_inputs(w, args.profile, args.latents)
     q, s, _ = oracle.cache.quantize_rows(x0)
     times = []
     for i in range(args.warmup + args.steps):
-        step_s, sample, _ = oracle_sample(w, audio, W, cond, xs[i % 2], q, s, rnum, rden)
+        step_s, sample, _ = oracle_sample(w, audio, W, cond, xs[i % 2], q, s, rnum, rden,
+                                          form=args.cache, selection=args.select, tau=args.tau,
+                                          seg_len=args.seg_len or None)
         if i >= args.warmup:
             times.append(step_s)
     ms = 1e3 * statistics.mean(times)
@@ -326,7 +358,11 @@ def run_sweep(args, w, blocks, x0, xs, dev, rank, world):
 
     profiles = w.sweep_profiles or (args.profile,)
     ratios = w.sweep_ratios or ((w.ratio_num, w.ratio_den),)
-    stack = CachedStack(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc, blocks, device=dev)
+    kinds = {"int8": ec.CACHE_INT8, "bf16": ec.CACHE_BF16, "ref": ec.CACHE_REF}
+    seg_len = args.seg_len or w.Wp
+    stack = CachedStack(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc, blocks, device=dev,
+                        cache_kind=kinds[args.cache], seg_len=seg_len, tau=args.tau,
+                        selection=args.select)
     x0_d = torch.from_numpy(x0).to(dev, torch.bfloat16)
     xs_d = [torch.from_numpy(x).to(dev, torch.bfloat16) for x in xs]
     stream = torch.cuda.current_stream()
@@ -414,7 +450,7 @@ def main():
         if world > 1:
             dist.barrier()
 
-    audio, W, cond, x0, xs = build_inputs(w, args.profile)
+    audio, W, cond, x0, xs = build_inputs(w, args.profile, args.latents)
     from synth import generate as G
     blocks = [ec.DeviceBlock.from_host(W if l == 0 else G.block_weights(w, l), cond, device=dev)
               for l in range(w.layers)]
@@ -504,13 +540,17 @@ def main():
                "h2d_bytes_per_step": xh[0].numel() * 2, "d2h_bytes_per_step": yh[0].numel() * 2,
                "ms_per_step": round(ems, 3)}
 
+    cache_bytes = stack.cache_bytes()
+    cache_bytes_rs = stack.cache_bytes(right_sized=True)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
         q, s, _ = oracle.cache.quantize_rows(x0)
         cr = (K, w.NT) if rate is not None else (rnum, rden)
         step_s, sample, _ = oracle_sample(w, audio, W, cond, xs[0], q, s, *cr,
-                                          adaptive=rate is not None)
+                                          adaptive=rate is not None, form=args.cache,
+                                          selection=args.select, tau=args.tau,
+                                          seg_len=args.seg_len or None)
         cpu = {"value": round(w.NT / step_s, 2), "unit": UNIT, "cores": cpu_cores(),
                "kind": "oracle", "sample": sample, "ms_per_step": round(step_s * 1e3, 1)}
 
@@ -524,9 +564,21 @@ def main():
                            "D": w.D, "heads": f"{w.H}x{w.d}",
                            "ffn": w.F, "audio_tokens": w.Lc, "layers": w.layers,
                            "audio": args.profile, "parallelism": f"replicas{world}",
+                           "cache": args.cache, "selection": args.select,
+                           "latents": args.latents,
                            "l2": "inputs larger than L2 (x 335 MB, weights 702 MB per block)"},
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
                 "gpu_launches": launches, "kernels": table}
+        if args.cache == "ref":
+            live, hw = stack.caches[-1].stats()
+            line["config"]["ref_cache"] = {
+                "tau": args.tau, "seg_len": seg_len, "live_references": live,
+                "pool_high_water": hw}
+        line["cache_bytes"] = {"allocated": cache_bytes,
+                               "right_sized": cache_bytes_rs,
+                               "note": "device bytes of every layer's cache after the timed "
+                                       "steps; right_sized counts a reference pool at its "
+                                       "high-water mark"}
         if rate is not None:
             line["config"]["adaptive"] = {
                 "r_min": rate.r_min, "r_max": rate.r_max, "alpha": rate.alpha,

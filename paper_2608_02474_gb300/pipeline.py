@@ -68,18 +68,36 @@ class AdaptiveRate:
 class CachedStack:
     def __init__(self, T: int, N: int, D: int, H: int, d: int, F: int, Lc: int,
                  blocks: list, device="cuda", lam: float = 0.1, xi: float = 1e-6,
-                 mode: int = ec.MODE_ENERGY_DRIFT):
+                 mode: int = ec.MODE_ENERGY_DRIFT, cache_kind: int = ec.CACHE_INT8,
+                 R_cap: int | None = None, seg_len: int = 1, tau: float = 0.9,
+                 selection: str = "energy", seed: int = 0):
+        """cache_kind: ec.CACHE_INT8 (plain int8), ec.CACHE_BF16 (full
+        precision) or ec.CACHE_REF (reference plus int8 residual, Sec. 3.4,
+        with R_cap, seg_len and tau).  selection: "energy" (the energy-guided
+        anchors of Sec. 3.3), or the ablations "uniform" and "random" (keys
+        drawn on the device from a generator seeded with `seed`)."""
+        if selection not in ("energy", "uniform", "random"):
+            raise ValueError(f"unknown selection {selection!r}")
         self.T, self.N, self.D = T, N, D
         self.NT = T * N
         self.dims = ec.BlockDims(T, N, D, H, d, F, Lc)
         self.blocks = blocks
         self.lam, self.xi, self.mode = lam, xi, mode
+        self.cache_kind, self.selection = cache_kind, selection
         dev = torch.device(device)
         L = len(blocks)
-        self.cache_q = [torch.zeros(self.NT, D, dtype=torch.int8, device=dev) for _ in range(L)]
-        self.cache_s = [torch.zeros(self.NT, dtype=torch.float32, device=dev) for _ in range(L)]
-        self.ws = torch.empty(ec.echo_workspace_size(self.dims, self.NT), dtype=torch.uint8,
-                              device=dev)
+        if cache_kind == ec.CACHE_INT8:
+            self.cache_q = [torch.zeros(self.NT, D, dtype=torch.int8, device=dev) for _ in range(L)]
+            self.cache_s = [torch.zeros(self.NT, dtype=torch.float32, device=dev) for _ in range(L)]
+            self.caches = None
+            ws = ec.echo_workspace_size(self.dims, self.NT)
+        else:
+            self.caches = [ec.DeviceCache(cache_kind, self.NT, D, R_cap=R_cap, seg_len=seg_len,
+                                          tau=tau, device=dev) for _ in range(L)]
+            ws = ec.echo_block_step_cache_workspace_size(self.dims, self.NT, self.caches[0])
+        self.ws = torch.empty(ws, dtype=torch.uint8, device=dev)
+        self.keys = torch.empty(self.NT, dtype=torch.float32, device=dev)
+        self.gen = torch.Generator(device=dev).manual_seed(seed)
         self.sel_ws = torch.empty(ec.echo_select_workspace_size(T, N), dtype=torch.uint8, device=dev)
         self.idx = torch.empty(self.NT, dtype=torch.int32, device=dev)
         self.all_idx = torch.arange(self.NT, dtype=torch.int32, device=dev)
@@ -105,18 +123,43 @@ class CachedStack:
         for l, blk in enumerate(self.blocks):
             if full:
                 idx, K = self.all_idx, self.NT
-            else:
+            elif self.selection == "uniform":
+                idx, K = ec.echo_select_uniform(self.T, self.N, ratio_num, ratio_den, idx=self.idx)
+            elif self.selection == "random":
+                torch.rand(self.NT, generator=self.gen, out=self.keys)
+                idx, K = ec.echo_select_random(self.keys, self.T, self.N, ratio_num, ratio_den,
+                                               idx=self.idx)
+            elif self.caches is None:
                 idx, K, _ = ec.echo_select(cur, self.cache_q[l], self.cache_s[l], self.seg, self.T,
                                            self.N, ratio_num, ratio_den, self.lam, self.xi,
                                            self.mode, idx=self.idx,
                                            scores=self.scores if keep_scores else None,
                                            workspace=self.sel_ws)
+            else:
+                idx, K, _ = ec.echo_select_cache(cur, self.caches[l], self.seg, self.T, self.N,
+                                                 ratio_num, ratio_den, self.lam, self.xi,
+                                                 self.mode, idx=self.idx,
+                                                 scores=self.scores if keep_scores else None,
+                                                 workspace=self.sel_ws)
             dst = out if (l == last and out is not None) else self.y[l % 2]
-            ec.echo_block_step(blk, self.dims, cur, idx, K, self.cache_q[l], self.cache_s[l],
-                               y=dst, workspace=self.ws)
+            if self.caches is None:
+                ec.echo_block_step(blk, self.dims, cur, idx, K, self.cache_q[l], self.cache_s[l],
+                                   y=dst, workspace=self.ws)
+            else:
+                ec.echo_block_step_cache(blk, self.dims, cur, idx, K, self.caches[l], y=dst,
+                                         workspace=self.ws)
             self.last_K.append(K)
             cur = dst
         return cur
+
+    def cache_bytes(self, right_sized: bool = False) -> int:
+        """Device bytes of every layer's cache; with right_sized, a reference
+        pool holds only the rows in use (its high-water mark; synchronises)."""
+        if self.caches is None:
+            return sum(q.numel() + 4 * s.numel() for q, s in zip(self.cache_q, self.cache_s))
+        if right_sized and self.cache_kind == ec.CACHE_REF:
+            return sum(c.nbytes(pool_rows=c.stats()[1]) for c in self.caches)
+        return sum(c.nbytes() for c in self.caches)
 
     def step_adaptive(self, x: torch.Tensor, rate: AdaptiveRate, full: bool = False,
                       keep_scores: bool = False, out: torch.Tensor | None = None) -> torch.Tensor:

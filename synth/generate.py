@@ -108,6 +108,18 @@ def latents(w: Workload) -> np.ndarray:
     return to_bf16_values(rng(1).standard_normal((w.NT, w.D), dtype=np.float32))
 
 
+def latents_smooth(w: Workload, rho: float = 0.95) -> np.ndarray:
+    """x0 with spatially adjacent tokens alike: along each row of W' tokens of
+    a latent frame the rows follow an AR(1) chain, x_w = rho x_{w-1} +
+    sqrt(1 - rho^2) e_w, e ~ N(0, 1) (seed 1), so neighbouring tokens have
+    cosine similarity about rho, as in real video latents.  [NT, D] bf16 values."""
+    e = rng(1).standard_normal((w.T * w.Hp, w.Wp, w.D), dtype=np.float32)
+    c = np.float32(np.sqrt(1.0 - rho * rho))
+    for k in range(1, w.Wp):
+        e[:, k] = np.float32(rho) * e[:, k - 1] + c * e[:, k]
+    return to_bf16_values(e.reshape(w.NT, w.D))
+
+
 def step_input(w: Workload, x0: np.ndarray, t: int) -> np.ndarray:
     """Layer-0 input at step t: bf16(x0 + sum_{s=1..t} eps_s), eps_s ~ N(0, 0.05^2)."""
     acc = x0.astype(np.float32).copy()
