@@ -4,12 +4,14 @@
 //
 // A REF write is four stream-ordered kernels:
 //   ref_release  every written token drops its old reference (atomic
-//                decrement of the slot's count);
+//                decrement of the slot's count) and the bounds of each scan
+//                segment's written rows are recorded;
 //   ref_scan     one CTA per scan segment walks its written rows in token
-//                order; its 8 warps test the next 8 rows against the current
-//                reference at once (fp32 cosine in the canonical order), the
-//                first row that fails becomes the new reference and the walk
-//                resumes after it;
+//                order, 8 rows a round: the rows are staged in shared memory,
+//                the 16 warps compute every fp32 cosine the walk can need (each
+//                row against the entering reference and against each earlier
+//                row of the round, canonical order), then one thread walks the
+//                8 rows and the last new reference carries into the next round;
 //   ref_alloc    one CTA ranks the new references in token order and hands
 //                them the free slots in slot order (block scans);
 //   ref_store    one warp per written row: a reference copies its row into its
@@ -21,7 +23,7 @@
 
 namespace {
 
-constexpr int kScanWarps = 8;
+constexpr int kScanWarps = 16;
 constexpr int kAllocThreads = 1024;
 constexpr int kStoreThreads = 256;
 constexpr int kVec = 256;
@@ -40,105 +42,162 @@ ECHO_DEV bool bf16_nonfinite(uint32_t two) {
 }
 
 // ---------------------------------------------------------------- release
-__global__ void ref_release_kernel(const int32_t *__restrict__ rows, int n,
-                                   const int32_t *__restrict__ ref, int32_t *refcount) {
+// every written token drops its reference (when a pool exists); the written
+// rows of scan segment s are positions [seg_lo[s], seg_hi[s]) of rows (seg_lo
+// stays -1 for a segment with none; rows ascending)
+__global__ void ref_release_kernel(const int32_t *__restrict__ rows, int n, int seg_len,
+                                   const int32_t *__restrict__ ref, int32_t *refcount,
+                                   int32_t *__restrict__ seg_lo, int32_t *__restrict__ seg_hi) {
     const int j = blockIdx.x * blockDim.x + threadIdx.x;
     if (j < n) {
-        const int old = ref[rows[j]];
-        if (old >= 0) atomicSub(&refcount[old], 1);
+        const int i = rows[j];
+        if (refcount) {
+            const int old = ref[i];
+            if (old >= 0) atomicSub(&refcount[old], 1);
+        }
+        const int sg = i / seg_len;
+        if (j == 0 || rows[j - 1] / seg_len != sg) seg_lo[sg] = j;
+        if (j == n - 1 || rows[j + 1] / seg_len != sg) seg_hi[sg] = j + 1;
     }
 }
 
 // ---------------------------------------------------------------- scan
-// fp32 cosine similarity of two bf16 rows, the three sums in the canonical
-// order (lane l owns 8-element chunks l, l+32, ...; chunk sums left to right;
-// xor butterfly 16..1).  Every lane returns the same value.
-ECHO_DEV float warp_cosine(const __nv_bfloat16 *a, const __nv_bfloat16 *b, int D, int lane) {
-    float dot = 0.f, na = 0.f, nb = 0.f;
-    const int C = D >> 3;
+// The canonical-order fp32 sums <a, b> (and <a, a> when `norm`) of two bf16
+// rows in shared memory: lane l owns 8-element chunks l, l+32, ..., adds each
+// chunk's sum left to right into its accumulator in chunk order, then an xor
+// butterfly 16..1.  Every lane returns the same sums.
+ECHO_DEV void warp_dot(const uint4 *a, const uint4 *b, int C, int lane, bool norm, float &dot,
+                       float &na) {
+    dot = 0.f;
+    na = 0.f;
     for (int c = lane; c < C; c += 32) {
         float fa[8], fb[8];
-        unpack8_bf16(*reinterpret_cast<const uint4 *>(a + 8 * c), fa);
-        unpack8_bf16(*reinterpret_cast<const uint4 *>(b + 8 * c), fb);
+        unpack8_bf16(a[c], fa);
+        unpack8_bf16(b[c], fb);
         float cd = __fmul_rn(fa[0], fb[0]);
-        float ca = __fmul_rn(fa[0], fa[0]);
-        float cb = __fmul_rn(fb[0], fb[0]);
+        float cn = __fmul_rn(fa[0], fa[0]);
 #pragma unroll
         for (int k = 1; k < 8; ++k) {
             cd = __fadd_rn(cd, __fmul_rn(fa[k], fb[k]));
-            ca = __fadd_rn(ca, __fmul_rn(fa[k], fa[k]));
-            cb = __fadd_rn(cb, __fmul_rn(fb[k], fb[k]));
+            if (norm) cn = __fadd_rn(cn, __fmul_rn(fa[k], fa[k]));
         }
         dot = __fadd_rn(dot, cd);
-        na = __fadd_rn(na, ca);
-        nb = __fadd_rn(nb, cb);
+        if (norm) na = __fadd_rn(na, cn);
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         dot = __fadd_rn(dot, __shfl_xor_sync(0xffffffffu, dot, o));
         na = __fadd_rn(na, __shfl_xor_sync(0xffffffffu, na, o));
-        nb = __fadd_rn(nb, __shfl_xor_sync(0xffffffffu, nb, o));
     }
-    if (!(na > 0.f) || !(nb > 0.f)) return 0.f;
-    return __fdiv_rn(dot, __fmul_rn(__fsqrt_rn(na), __fsqrt_rn(nb)));
 }
 
-ECHO_DEV int lower_bound(const int32_t *v, int n, int key) {
-    int lo = 0, hi = n;
-    while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if (v[mid] < key) lo = mid + 1;
-        else hi = mid;
-    }
-    return lo;
-}
+// src_pos[j] = position (in rows) of row j's reference; j itself for a reference.
+//
+// One CTA per scan segment.  The segment's written rows are taken kWin at a
+// time: the window's rows are staged in shared memory, then the CTA computes
+// every similarity the walk over the window can need (each row against the
+// reference it entered with and against every earlier row of the window), and
+// one thread walks the window in order.  A window is resolved in one round
+// whatever the data.  Dynamic shared memory: kWin window rows, then the
+// current reference row (bf16, D each).
+constexpr int kWin = 8;
+constexpr int kPairs = kWin * (kWin + 1) / 2;
 
-// src_pos[j] = position (in rows) of row j's reference; j itself for a reference
 __global__ void __launch_bounds__(kScanWarps * 32)
-ref_scan_kernel(const __nv_bfloat16 *__restrict__ src, const int32_t *__restrict__ rows, int n,
-                int seg_len, float tau, int D, int32_t *__restrict__ src_pos) {
-    __shared__ int s_lo, s_hi, s_j, s_jr;
-    __shared__ int s_pass[kScanWarps];
+ref_scan_kernel(const __nv_bfloat16 *__restrict__ src, const int32_t *__restrict__ seg_lo,
+                const int32_t *__restrict__ seg_hi, float tau, int D,
+                int32_t *__restrict__ src_pos) {
+    extern __shared__ uint4 s_buf[];
+    __shared__ float s_dot[kWin][kWin + 1];  // [w][t + 1], t = -1: the entering reference
+    __shared__ float s_nv[kWin];
+    __shared__ float s_nr;
+    __shared__ int s_jr, s_newref;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int C = D >> 3;
+    uint4 *ref = s_buf + (size_t)kWin * C;
+    const int lo = seg_lo[blockIdx.x];
+    if (lo < 0) return;
+    const int hi = seg_hi[blockIdx.x];
     if (threadIdx.x == 0) {
-        const int64_t first = (int64_t)blockIdx.x * seg_len;
-        const int64_t last = first + seg_len;
-        s_lo = lower_bound(rows, n, (int)first);
-        s_hi = lower_bound(rows, n, (int)(last < INT32_MAX ? last : INT32_MAX));
-        if (s_lo < s_hi) src_pos[s_lo] = s_lo;
-        s_jr = s_lo;
-        s_j = s_lo + 1;
+        src_pos[lo] = lo;
+        s_jr = lo;
+    }
+    // the segment's first written row is its first reference
+    {
+        const uint4 *v = reinterpret_cast<const uint4 *>(src + (int64_t)lo * D);
+        for (int c = threadIdx.x; c < C; c += blockDim.x) ref[c] = __ldg(v + c);
     }
     __syncthreads();
-    const int hi = s_hi;
-    if (s_lo >= hi) return;
-    // every iteration consumes at least one row, so at most hi - lo iterations
-    while (true) {
-        const int j = s_j, jr = s_jr;
-        if (j >= hi) break;
-        const int jj = j + warp;
-        if (jj < hi) {
-            const float sim = warp_cosine(src + (int64_t)jj * D, src + (int64_t)jr * D, D, lane);
-            if (lane == 0) s_pass[warp] = sim > tau ? 1 : 0;
+    if (warp == 0) {
+        float d, nr;
+        warp_dot(ref, ref, C, lane, true, d, nr);
+        if (lane == 0) s_nr = nr;
+    }
+    __syncthreads();
+    for (int j = lo + 1; j < hi; j += kWin) {
+        const int nvalid = hi - j < kWin ? hi - j : kWin;
+        // stage the window's rows, four 16-byte loads in flight per thread
+        const int total = nvalid * C;
+        for (int b = threadIdx.x; b < total; b += 4 * (int)blockDim.x) {
+            uint4 u[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int e = b + k * blockDim.x;
+                if (e < total) {
+                    const int w = e / C, c = e - w * C;
+                    u[k] = __ldg(reinterpret_cast<const uint4 *>(src + (int64_t)(j + w) * D) + c);
+                }
+            }
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int e = b + k * blockDim.x;
+                if (e < total) s_buf[e] = u[k];
+            }
+        }
+        __syncthreads();
+        // pair p = (w, t): row w of the window against t = -1 (the entering
+        // reference) or the earlier window row t; pairs of row w start at w(w+1)/2
+        for (int p = warp; p < kPairs; p += kScanWarps) {
+            int w = 0;
+            while ((w + 1) * (w + 2) / 2 <= p) ++w;
+            const int t = p - w * (w + 1) / 2 - 1;
+            if (w >= nvalid) continue;
+            float dot, nv;
+            warp_dot(s_buf + (size_t)w * C, t < 0 ? ref : s_buf + (size_t)t * C, C, lane, t < 0,
+                     dot, nv);
+            if (lane == 0) {
+                s_dot[w][t + 1] = dot;
+                if (t < 0) s_nv[w] = nv;
+            }
         }
         __syncthreads();
         if (threadIdx.x == 0) {
-            const int nvalid = hi - j < kScanWarps ? hi - j : kScanWarps;
-            int f = nvalid;
-            for (int w = 0; w < nvalid; ++w)
-                if (!s_pass[w]) {
-                    f = w;
-                    break;
+            int cur = -1;
+            float ncur = s_nr;
+            const int jr = s_jr;
+            for (int w = 0; w < nvalid; ++w) {
+                const float nv = s_nv[w];
+                float sim = 0.f;
+                if (nv > 0.f && ncur > 0.f)
+                    sim = __fdiv_rn(s_dot[w][cur + 1], __fmul_rn(__fsqrt_rn(nv), __fsqrt_rn(ncur)));
+                if (sim > tau) {
+                    src_pos[j + w] = cur < 0 ? jr : j + cur;
+                } else {
+                    src_pos[j + w] = j + w;
+                    cur = w;
+                    ncur = nv;
                 }
-            for (int w = 0; w < f; ++w) src_pos[j + w] = jr;
-            if (f < nvalid) {
-                src_pos[j + f] = j + f;
-                s_jr = j + f;
-                s_j = j + f + 1;
-            } else {
-                s_j = j + nvalid;
+            }
+            s_newref = cur;
+            if (cur >= 0) {
+                s_jr = j + cur;
+                s_nr = ncur;
             }
         }
+        __syncthreads();
+        const int nr = s_newref;
+        if (nr >= 0)
+            for (int c = threadIdx.x; c < C; c += blockDim.x) ref[c] = s_buf[(size_t)nr * C + c];
         __syncthreads();
     }
 }
@@ -418,19 +477,26 @@ __global__ void cache_stats_kernel(const int32_t *__restrict__ refcount, int R_c
 }
 
 struct RefWs {
-    int32_t *src_pos, *slot_of, *free_list;
+    int32_t *src_pos, *slot_of, *free_list, *seg_lo, *seg_hi;
 };
 
-size_t ref_ws_bytes(int32_t n) {
-    const size_t a = al256(sizeof(int32_t) * (size_t)(n > 0 ? n : 1));
-    return 3 * a;
+int n_segments(const echo_cache &c) {
+    return (int)((c.NT + (int64_t)c.seg_len - 1) / c.seg_len);
 }
 
-RefWs ref_ws(void *ws, int32_t n) {
+size_t ref_ws_bytes(const echo_cache &c, int32_t n) {
     const size_t a = al256(sizeof(int32_t) * (size_t)(n > 0 ? n : 1));
-    uint8_t *b = static_cast<uint8_t *>(ws);
-    return {reinterpret_cast<int32_t *>(b), reinterpret_cast<int32_t *>(b + a),
-            reinterpret_cast<int32_t *>(b + 2 * a)};
+    const size_t b = al256(sizeof(int32_t) * (size_t)n_segments(c));
+    return 3 * a + 2 * b;
+}
+
+RefWs ref_ws(const echo_cache &c, void *ws, int32_t n) {
+    const size_t a = al256(sizeof(int32_t) * (size_t)(n > 0 ? n : 1));
+    const size_t b = al256(sizeof(int32_t) * (size_t)n_segments(c));
+    uint8_t *p = static_cast<uint8_t *>(ws);
+    return {reinterpret_cast<int32_t *>(p), reinterpret_cast<int32_t *>(p + a),
+            reinterpret_cast<int32_t *>(p + 2 * a), reinterpret_cast<int32_t *>(p + 3 * a),
+            reinterpret_cast<int32_t *>(p + 3 * a + b)};
 }
 
 }  // namespace
@@ -463,7 +529,7 @@ echo_status cache_check(const echo_cache *c) {
 }
 
 size_t cache_write_ws(const echo_cache &c, int32_t n) {
-    return c.kind == ECHO_CACHE_REF ? ref_ws_bytes(n) : 0;
+    return c.kind == ECHO_CACHE_REF ? ref_ws_bytes(c, n) : 0;
 }
 
 echo_status launch_cache_write(const echo_cache &c, const void *src, const int32_t *rows,
@@ -481,17 +547,25 @@ echo_status launch_cache_write(const echo_cache &c, const void *src, const int32
             s, rows, n, c.D, static_cast<__nv_bfloat16 *>(c.full), err);
         return last_launch_status();
     }
-    const RefWs w = ref_ws(ws, n);
-    if (c.R_cap > 0) {
+    const RefWs w = ref_ws(c, ws, n);
+    const int nseg = n_segments(c);
+    if (cudaMemsetAsync(w.seg_lo, 0xFF, sizeof(int32_t) * (size_t)nseg, st) != cudaSuccess)
+        return ECHO_ERR_CUDA;
+    {
         LaunchScope ls(ECHO_K_REF_ALLOC, n, c.D, 0, st);
-        ref_release_kernel<<<(n + 255) / 256, 256, 0, st>>>(rows, n, c.ref, c.refcount);
+        ref_release_kernel<<<(n + 255) / 256, 256, 0, st>>>(
+            rows, n, c.seg_len, c.ref, c.R_cap > 0 ? c.refcount : nullptr, w.seg_lo, w.seg_hi);
     }
     if (last_launch_status() != ECHO_OK) return ECHO_ERR_CUDA;
-    const int nseg = (int)((c.NT + (int64_t)c.seg_len - 1) / c.seg_len);
     {
+        const size_t smem = (size_t)(kWin + 1) * c.D * sizeof(__nv_bfloat16);
+        if (smem > 48 * 1024 &&
+            cudaFuncSetAttribute(ref_scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)smem) != cudaSuccess)
+            return ECHO_ERR_CUDA;
         LaunchScope ls(ECHO_K_REF_SCAN, n, c.D, 0, st);
-        ref_scan_kernel<<<nseg, kScanWarps * 32, 0, st>>>(s, rows, n, c.seg_len, c.tau, c.D,
-                                                          w.src_pos);
+        ref_scan_kernel<<<nseg, kScanWarps * 32, smem, st>>>(s, w.seg_lo, w.seg_hi, c.tau, c.D,
+                                                             w.src_pos);
     }
     if (last_launch_status() != ECHO_OK) return ECHO_ERR_CUDA;
     {

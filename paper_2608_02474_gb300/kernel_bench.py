@@ -25,7 +25,7 @@ def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--kernel", required=True,
                     choices=["gemm", "attention", "drift", "select", "merge", "quant", "layernorm",
-                             "energy", "step_delta"])
+                             "energy", "step_delta", "ref_write"])
     ap.add_argument("--M", type=int, default=6552)
     ap.add_argument("--N", type=int, default=5120)
     ap.add_argument("--K", type=int, default=5120)
@@ -102,6 +102,24 @@ def main():
         ws = torch.empty(ec.echo_step_delta_workspace_size(n), dtype=torch.uint8, device=dev)
         run = lambda: ec.echo_step_delta(hp, hc, out=out, workspace=ws)
         work, unit = 4.0 * n, "GB/s"
+    elif a.kernel == "ref_write":
+        # reference-plus-residual cache write of K rows (scan segments of 52
+        # tokens, tau 0.9) into a cache filled with rows alike along the token
+        # order; the rows written are alike too (AR(1), rho 0.95)
+        NT, D = a.T * a.N, a.D
+        # AR(1) along the token order within each run of 52 tokens
+        x = rn(NT, D)
+        x = x.view(-1, 52, D) if NT % 52 == 0 else x.view(1, NT, D)
+        for k in range(1, x.shape[1]):
+            x[:, k] = 0.95 * x[:, k - 1] + (1 - 0.95 ** 2) ** 0.5 * x[:, k]
+        full = x.reshape(NT, D).to(torch.bfloat16)
+        cache = ec.DeviceCache(ec.CACHE_REF, NT, D, seg_len=52, tau=0.9, device=dev)
+        cache.write(full, torch.arange(NT, dtype=torch.int32, device=dev))
+        rows = torch.sort(torch.randperm(NT, generator=g, device=dev)[:a.K]).values.to(torch.int32)
+        src = full[rows.long()].contiguous()
+        ws = torch.empty(cache.write_workspace_size(a.K), dtype=torch.uint8, device=dev)
+        run = lambda: cache.write(src, rows, workspace=ws)
+        work, unit = a.K * (3.0 * D + 8), "GB/s"
     elif a.kernel == "energy":
         audio = rn(a.samples)
         band = torch.empty(a.T, 8, dtype=torch.float32, device=dev)
