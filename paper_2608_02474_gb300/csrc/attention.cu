@@ -134,6 +134,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer ----------------
         // order: S0_0 S1_0 | PV0_0 S0_1 PV1_0 S1_1 | PV0_1 S0_2 PV1_1 S1_2 | ...
+        // Each ring slot is waited for once, before tile 0 uses it: a wait costs
+        // about as much as an MMA even when the data has landed, and this thread
+        // issues tile 1's use of the same slot later.
         // P_t lives in the first 64 columns of S_t; S_t of the next block is
         // issued after P V of this block, and tcgen05.mma from one thread run in
         // order, so the S write cannot overtake the P read.  The commit of S_t
@@ -141,8 +144,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         bool ok = mbar_wait(&q_full, 0, abort_v, p.err);
         auto issue_s = [&](int t, int j) -> bool {
             const int li = 2 * j, slot = li % RING;
-            if (!mbar_wait(&ring_full[slot], (li / RING) & 1, abort_v, p.err)) return false;
-            tc_fence_after();
+            if (t == 0) {   // tile 1 uses the slot after tile 0: this thread saw it land
+                if (!mbar_wait(&ring_full[slot], (li / RING) & 1, abort_v, p.err)) return false;
+                tc_fence_after();
+            }
             const uint8_t *qt = Qs + t * C::Q_BYTES;
             const uint8_t *kt = Ring + slot * C::SLOT_BYTES;
 #pragma unroll
@@ -158,7 +163,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         auto issue_pv = [&](int t, int j) -> bool {
             const int li = 2 * j + 1, slot = li % RING;
             if (!mbar_wait(&p_full[t], j & 1, abort_v, p.err)) return false;
-            if (!mbar_wait(&ring_full[slot], (li / RING) & 1, abort_v, p.err)) return false;
+            if (t == 0 && !mbar_wait(&ring_full[slot], (li / RING) & 1, abort_v, p.err)) return false;
             tc_fence_after();
             const uint8_t *vt = Ring + slot * C::SLOT_BYTES;
 #pragma unroll
