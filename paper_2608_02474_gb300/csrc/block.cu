@@ -13,8 +13,9 @@
 //   attention   att = MHA(Qc, Kc, Vc)
 //   GEMM        h2 = att Woc^T + boc + h1               (fp32)
 //   LN, GEMM    u = GELU(LN(h2) W1^T + b1)
-//   GEMM        y_act = u W2^T + b2 + h2                (bf16)
-//   quant       cache[idx] = Q(y_act)
+//   GEMM        y_act = u W2^T + b2 + h2                (bf16; the epilogue
+//               also folds max |y_act| per row for the quantiser)
+//   quant       cache[idx] = Q(y_act)                   (one pass over y_act)
 //   merge       y = fresh rows at idx, reconstructed cache elsewhere
 #include "common.cuh"
 #include "internal.h"
@@ -24,7 +25,7 @@ namespace {
 size_t al(size_t b) { return (b + 255) & ~(size_t)255; }
 
 struct Layout {
-    size_t rowmap, n1, kv, na, qa, att, h1, h2, u, yact, total;
+    size_t rowmap, n1, kv, na, qa, att, h1, h2, u, yact, amax, total;
 };
 
 Layout layout(const echo_block_dims &d, int64_t K) {
@@ -41,6 +42,7 @@ Layout layout(const echo_block_dims &d, int64_t K) {
     L.h2 = o;     o += al(4 * (size_t)K * d.D);
     L.u = o;      o += al(2 * (size_t)K * d.F);
     L.yact = o;   o += al(2 * (size_t)K * d.D);
+    L.amax = o;   o += al(4 * (size_t)K);
     L.total = o;
     return L;
 }
@@ -130,8 +132,14 @@ echo_status run_active(const echo_block_weights *w, const echo_block_dims &d, co
         s = launch_linear({na, D, K, D, w->W1, w->b1, d.F, 1, nullptr, ECHO_BF16, nullptr, u, d.F,
                            ECHO_BF16}, st);
         if (s != ECHO_OK) return s;
-        s = launch_linear({u, d.F, K, d.F, w->W2, w->b2, D, 0, h2, ECHO_F32, nullptr, yact, D,
-                           ECHO_BF16}, st);
+        // the FFN-down epilogue also records max |y_act| per row for the cache write
+        uint32_t *amax = reinterpret_cast<uint32_t *>(ws + L.amax);
+        if (cudaMemsetAsync(amax, 0, sizeof(uint32_t) * (size_t)K, st) != cudaSuccess)
+            return ECHO_ERR_CUDA;
+        LinearArgs down{u, d.F, K, d.F, w->W2, w->b2, D, 0, h2, ECHO_F32, nullptr, yact, D,
+                        ECHO_BF16};
+        down.row_amax = amax;
+        s = launch_linear(down, st);
         if (s != ECHO_OK) return s;
     }
     return last_launch_status();
@@ -161,7 +169,9 @@ extern "C" echo_status echo_block_step(const echo_block_weights *w, const echo_b
     // the merge reads the cache of the inactive rows only, the quantiser writes
     // the active rows only: their order does not matter
     launch_dequant_merge(cache_q, cache_scale, rowmap, ws + L.yact, NT, d.D, y, st);
-    if (K > 0) launch_quant(ws + L.yact, ECHO_BF16, idx, K, d.D, cache_q, cache_scale, st);
+    if (K > 0)
+        launch_quant_amax(ws + L.yact, reinterpret_cast<const uint32_t *>(ws + L.amax), idx, K,
+                          d.D, cache_q, cache_scale, st);
     return last_launch_status();
 }
 

@@ -88,6 +88,51 @@ quant_kernel(const ST *__restrict__ src, const int32_t *__restrict__ rows, int n
     }
 }
 
+// quant_kernel with the row's max |v| given (computed where the rows were
+// produced): one read of each row.  Same rules and the same bits.
+__global__ void __launch_bounds__(kQuantThreads)
+quant_amax_kernel(const __nv_bfloat16 *__restrict__ src, const uint32_t *__restrict__ amax_bits,
+                  const int32_t *__restrict__ rows, int n_rows, int D, int8_t *__restrict__ q,
+                  float *__restrict__ scale, int *err) {
+    const int lane = threadIdx.x & 31;
+    const int warps = blockDim.x >> 5;
+    const int C = D >> 3;
+    for (int j = blockIdx.x * warps + (threadIdx.x >> 5); j < n_rows; j += gridDim.x * warps) {
+        const __nv_bfloat16 *s = src + (int64_t)j * D;
+        const uint32_t ab = amax_bits[j];
+        const float amax = __uint_as_float(ab);
+        const int r = rows ? rows[j] : j;
+        int8_t *qr = q + (int64_t)r * D;
+        if (ab >= 0x7F800000u) {   // NaN or infinity in the row
+            for (int c = lane; c < C; c += 32) *reinterpret_cast<uint2 *>(qr + 8 * c) = make_uint2(0, 0);
+            if (lane == 0) {
+                scale[r] = ab > 0x7F800000u ? __int_as_float(0x7fc00000) : INFINITY;
+                echo_flag_error(err, ECHO_ERR_NONFINITE);
+            }
+            continue;
+        }
+        float sc = 0.f, inv = 0.f;
+        if (amax > 0.f) {
+            sc = __fdiv_rn(amax, 127.f);
+            inv = __fdiv_rn(127.f, amax);
+        }
+        for (int c = lane; c < C; c += 32) {
+            float f[8];
+            load8<__nv_bfloat16>(s + 8 * c, f);
+            uint32_t w[2] = {0u, 0u};
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                float t = rintf(__fmul_rn(f[k], inv));
+                t = fminf(fmaxf(t, -127.f), 127.f);
+                const uint32_t b = (uint32_t)(uint8_t)(int8_t)(int)t;
+                w[k >> 2] |= b << (8 * (k & 3));
+            }
+            *reinterpret_cast<uint2 *>(qr + 8 * c) = make_uint2(w[0], w[1]);
+        }
+        if (lane == 0) scale[r] = sc;
+    }
+}
+
 ECHO_DEV void dequant16(const int4 &qv, float s, float *f) {
     const int8_t *b = reinterpret_cast<const int8_t *>(&qv);
 #pragma unroll
@@ -185,6 +230,16 @@ void launch_quant(const void *src, echo_dtype st_t, const int32_t *rows, int32_t
     else
         quant_kernel<float><<<grid, kQuantThreads, 0, st>>>(static_cast<const float *>(src), rows,
                                                             n_rows, D, q, scale, err);
+}
+
+void launch_quant_amax(const void *src, const uint32_t *amax, const int32_t *rows, int32_t n_rows,
+                       int32_t D, int8_t *q, float *scale, cudaStream_t st) {
+    if (n_rows <= 0) return;
+    const int grid = grid_for((int64_t)n_rows * 32, kQuantThreads);
+    LaunchScope ls(ECHO_K_QUANT, n_rows, D, 0, st);
+    quant_amax_kernel<<<grid, kQuantThreads, 0, st>>>(static_cast<const __nv_bfloat16 *>(src), amax,
+                                                      rows, n_rows, D, q, scale,
+                                                      device_error_ptr());
 }
 
 void launch_dequant(const int8_t *q, const float *scale, const int32_t *rows, int32_t n_rows,

@@ -30,7 +30,9 @@ constexpr uint32_t TMEM_COLS = 512;   // two 256-column accumulators
 constexpr int GROUP_N = 16;            // N tiles per raster band
 constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
 
-enum : int { EPI_GELU = 1, EPI_RES_BF16 = 2, EPI_RES_F32 = 4, EPI_OUT_F32 = 8 };
+// EPI_ROWAMAX: also fold max |v| of each bf16 output row into row_amax (fp32
+// bits, atomic max over the row's column tiles; a NaN beats every number)
+enum : int { EPI_GELU = 1, EPI_RES_BF16 = 2, EPI_RES_F32 = 4, EPI_OUT_F32 = 8, EPI_ROWAMAX = 16 };
 
 struct GemmParams {
     int M, N, Kd;
@@ -39,6 +41,7 @@ struct GemmParams {
     const int32_t *resid_rows;
     void *out;
     int64_t ldo;
+    uint32_t *row_amax;
     int *err;
 };
 
@@ -173,6 +176,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
             const bool row_ok = row < p.M;
             int rrow = row;
             if ((EPI & EPI_RES_BF16) && p.resid_rows && row_ok) rrow = p.resid_rows[row];
+            uint32_t rmax = 0;   // EPI_ROWAMAX: max |v| of this row's stored values, as bits
             for (int c = 0; c < BN; c += 32) {
                 const int col = n0 + c;
                 if (col >= p.N) break;                       // warp-uniform
@@ -225,9 +229,19 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                     uint4 *op = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.out) +
                                                           (int64_t)row * p.ldo + col);
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) op[i] = pack8_bf16(v + 8 * i);
+                    for (int i = 0; i < 4; ++i) {
+                        const uint4 pk = pack8_bf16(v + 8 * i);
+                        op[i] = pk;
+                        if (EPI & EPI_ROWAMAX) {
+                            const uint32_t w[4] = {pk.x, pk.y, pk.z, pk.w};
+#pragma unroll
+                            for (int e = 0; e < 4; ++e)
+                                rmax = max(rmax, max((w[e] & 0x7FFFu) << 16, w[e] & 0x7FFF0000u));
+                        }
+                    }
                 }
             }
+            if ((EPI & EPI_ROWAMAX) && row_ok) atomicMax(&p.row_amax[row], rmax);
             tc_fence_before();
             mbar_arrive(&acc_empty[buf]);
         }
@@ -287,11 +301,16 @@ echo_status launch_linear(const LinearArgs &a, cudaStream_t st) {
     p.resid_rows = a.resid_rows;
     p.out = a.out;
     p.ldo = a.ldo;
+    p.row_amax = a.row_amax;
     p.err = device_error_ptr();
     int epi = 0;
     if (a.act == 1) epi |= EPI_GELU;
     if (a.resid) epi |= (a.resid_t == ECHO_BF16) ? EPI_RES_BF16 : EPI_RES_F32;
     if (a.out_t == ECHO_F32) epi |= EPI_OUT_F32;
+    if (a.row_amax) {
+        if (epi != EPI_RES_F32) return ECHO_ERR_INVALID_ARG;   // bf16 out, fp32 residual only
+        return run<EPI_RES_F32 | EPI_ROWAMAX>(ta, tb, p, st);
+    }
     switch (epi) {
         case 0: return run<0>(ta, tb, p, st);
         case EPI_GELU: return run<EPI_GELU>(ta, tb, p, st);

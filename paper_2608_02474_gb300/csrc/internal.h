@@ -50,6 +50,7 @@ struct LinearArgs {
     const void *W; const void *bias; int32_t N; int32_t act;
     const void *resid; echo_dtype resid_t; const int32_t *resid_rows;
     void *out; int64_t ldo; echo_dtype out_t;
+    uint32_t *row_amax = nullptr;   // bf16 out with an fp32 residual only: max |out| per row
 };
 echo_status launch_linear(const LinearArgs &a, cudaStream_t st);
 
@@ -61,6 +62,9 @@ echo_status launch_attention(const void *Q, int64_t ldq, const void *K, const vo
 // cache.cu
 void launch_quant(const void *src, echo_dtype st_t, const int32_t *rows, int32_t n_rows,
                   int32_t D, int8_t *q, float *scale, cudaStream_t st);
+// int8 quantisation of bf16 rows whose max |v| is already known (fp32 bits)
+void launch_quant_amax(const void *src, const uint32_t *amax, const int32_t *rows, int32_t n_rows,
+                       int32_t D, int8_t *q, float *scale, cudaStream_t st);
 void launch_dequant(const int8_t *q, const float *scale, const int32_t *rows, int32_t n_rows,
                     int32_t D, void *dst, echo_dtype dt, cudaStream_t st);
 void launch_rowmap(const int32_t *idx, int32_t K, int32_t NT, int32_t *rowmap, cudaStream_t st);

@@ -184,6 +184,29 @@ def test_select_ties_take_lowest_index(ec):
     assert list(idx.cpu().numpy()) == list(range(K))
 
 
+def test_select_with_and_without_workspace_agree(ec):
+    """Scores kept by the caller, in the workspace, or both: the same selection,
+    equal to the oracle's, on a case with many equal scores (quantised energy,
+    repeated rows)."""
+    T, N, D = 21, 520, 128
+    NT = T * N
+    x = G.random_rows(NT, D, seed=41)
+    x[::3] = x[0]
+    q, s = G.random_cache(NT, D, seed=42)
+    q[::3], s[::3] = q[0], s[0]
+    e = np.floor(G.random_energy(T, seed=43) * 4).astype(F32)
+    qd = torch.from_numpy(q).to(DEV)
+    ws = torch.empty(ec.echo_select_workspace_size(T, N), dtype=torch.uint8, device=DEV)
+    sc = torch.empty(NT, dtype=torch.float32, device=DEV)
+    a, K, _ = ec.echo_select(bf(x), qd, f32(s), f32(e), T, N, 1, 5, scores=sc)
+    b, _, _ = ec.echo_select(bf(x), qd, f32(s), f32(e), T, N, 1, 5, scores=sc, workspace=ws)
+    c, _, _ = ec.echo_select(bf(x), qd, f32(s), f32(e), T, N, 1, 5, workspace=ws)
+    oidx, _ = oracle.select.select(x, q, s, e, T, N, 1, 5)
+    for r in (a, b, c):
+        assert np.array_equal(r.cpu().numpy(), oidx)
+    no_device_error(ec)
+
+
 def test_select_with_silence_is_drift_only(ec):
     T, N, D = 4, 64, 128
     x = G.random_rows(T * N, D, seed=5)
