@@ -3,9 +3,9 @@
 // stream-ordered kernels over a caller-owned workspace:
 //
 //   rowmap      token -> position in idx (or -1)
-//   LN          n1 = LN(x), all NT rows
+//   LN          n1 = LN(x), all NT rows; the active rows are also written to
+//               na = LN(x[idx]) through the row map  ("select active latents")
 //   GEMM        KV = n1 [Wk; Wv]^T + [bk; bv]          (K, V over all latents)
-//   LN+gather   na = LN(x[idx])                         ("select active latents")
 //   GEMM        Q' = na Wq^T + bq
 //   attention   att = MHA(Q', K, V)
 //   GEMM        h1 = att Wo^T + bo + x[idx]             (fp32)
@@ -107,11 +107,11 @@ echo_status run_active(const echo_block_weights *w, const echo_block_dims &d, co
     echo_status s = ECHO_OK;
     launch_rowmap(idx, K, NT, rowmap, st);
     if (K > 0) {
-        launch_layernorm(x, ECHO_BF16, nullptr, NT, D, n1, st);
+        // LN over every latent; the active rows also land in na, gathered
+        launch_layernorm_scatter(x, NT, D, n1, rowmap, na, st);
         s = launch_linear({n1, D, NT, D, w->Wkv, w->bkv, 2 * D, 0, nullptr, ECHO_BF16, nullptr, kv,
                            2 * (int64_t)D, ECHO_BF16}, st);
         if (s != ECHO_OK) return s;
-        launch_layernorm(x, ECHO_BF16, idx, K, D, na, st);
         s = launch_linear({na, D, K, D, w->Wq, w->bq, D, 0, nullptr, ECHO_BF16, nullptr, qa, D,
                            ECHO_BF16}, st);
         if (s != ECHO_OK) return s;

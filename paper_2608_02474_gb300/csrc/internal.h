@@ -43,6 +43,9 @@ bool make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t co
 // layernorm.cu
 void launch_layernorm(const void *in, echo_dtype in_t, const int32_t *rows, int32_t n_rows,
                       int32_t D, void *out, cudaStream_t st);
+// out = LN(in) for all n_rows bf16 rows; row i also goes to out2[map[i]] when map[i] >= 0
+void launch_layernorm_scatter(const void *in, int32_t n_rows, int32_t D, void *out,
+                              const int32_t *scatter_map, void *out2, cudaStream_t st);
 
 // gemm.cu: out = act(A W^T + bias) + resid
 struct LinearArgs {

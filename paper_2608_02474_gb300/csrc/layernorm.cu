@@ -1,6 +1,7 @@
 // Layer norm without affine, eps 1e-6, biased variance (the block's LN), with
-// an optional row gather: out[j] = LN(in[rows[j]]).  The gathered form is the
-// "select active latents" step of Sec. 3.3 fused with the LN that follows it.
+// an optional row gather: out[j] = LN(in[rows[j]]), or, for every row of a bf16
+// input, a second copy of the rows a map selects (the "select active latents"
+// step of Sec. 3.3 fused with the LN over all latents that the K/V path needs).
 //
 // A row lives in registers: for bf16 input one warp per row holds it packed (up
 // to 32 16-byte chunks per lane); for fp32 input up to 8 chunks of 8 values per
@@ -108,10 +109,14 @@ layernorm_kernel(const T *__restrict__ in, const int32_t *__restrict__ rows, int
 // bf16 input: one warp per row, the row held packed in registers (CPL 16-byte
 // chunks per lane), so each row is read from HBM once and no block barrier is
 // needed.
+// With scatter_map, row j is also written to out2[scatter_map[j]] when that is
+// >= 0: the LN of every latent (for K and V) then also yields the gathered LN
+// of the active ones (for Q') without reading them a second time.
 template <int CPL>
 __global__ void __launch_bounds__(kThreads)
 layernorm_warp_bf16(const __nv_bfloat16 *__restrict__ in, const int32_t *__restrict__ rows,
-                    int n_rows, int D, __nv_bfloat16 *__restrict__ out) {
+                    int n_rows, int D, __nv_bfloat16 *__restrict__ out,
+                    const int32_t *__restrict__ scatter_map, __nv_bfloat16 *__restrict__ out2) {
     const int lane = threadIdx.x & 31;
     const int warps = kThreads / 32;
     const int C = D >> 3;
@@ -153,6 +158,8 @@ layernorm_warp_bf16(const __nv_bfloat16 *__restrict__ in, const int32_t *__restr
         for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
         const float rstd = rsqrtf(ss * invD + 1e-6f);
         uint4 *dst = reinterpret_cast<uint4 *>(out + (int64_t)j * D);
+        const int j2 = scatter_map ? scatter_map[j] : -1;
+        uint4 *dst2 = j2 >= 0 ? reinterpret_cast<uint4 *>(out2 + (int64_t)j2 * D) : nullptr;
 #pragma unroll
         for (int k = 0; k < CPL; ++k) {
             const int c = lane + 32 * k;
@@ -161,7 +168,9 @@ layernorm_warp_bf16(const __nv_bfloat16 *__restrict__ in, const int32_t *__restr
                 unpack8_bf16(v[k], f);
 #pragma unroll
                 for (int e = 0; e < 8; ++e) f[e] = (f[e] - mean) * rstd;
-                dst[c] = pack8_bf16(f);
+                const uint4 o = pack8_bf16(f);
+                dst[c] = o;
+                if (dst2) dst2[c] = o;
             }
         }
     }
@@ -169,11 +178,25 @@ layernorm_warp_bf16(const __nv_bfloat16 *__restrict__ in, const int32_t *__restr
 
 template <int CPL>
 void launch_warp_bf16(const __nv_bfloat16 *in, const int32_t *rows, int n_rows, int D,
-                      __nv_bfloat16 *out, cudaStream_t st) {
+                      __nv_bfloat16 *out, const int32_t *scatter_map, __nv_bfloat16 *out2,
+                      cudaStream_t st) {
     constexpr int RPB = kThreads / 32;
     int grid = (n_rows + RPB - 1) / RPB;
     if (grid > 152 * 8) grid = 152 * 8;
-    layernorm_warp_bf16<CPL><<<grid, kThreads, 0, st>>>(in, rows, n_rows, D, out);
+    layernorm_warp_bf16<CPL><<<grid, kThreads, 0, st>>>(in, rows, n_rows, D, out, scatter_map,
+                                                        out2);
+}
+
+void launch_bf16(const __nv_bfloat16 *in, const int32_t *rows, int n_rows, int D,
+                 __nv_bfloat16 *out, const int32_t *scatter_map, __nv_bfloat16 *out2,
+                 cudaStream_t st) {
+    const int cpl = (D / 8 + 31) / 32;   // 16-byte chunks per lane
+    if (cpl <= 4) return launch_warp_bf16<4>(in, rows, n_rows, D, out, scatter_map, out2, st);
+    if (cpl <= 8) return launch_warp_bf16<8>(in, rows, n_rows, D, out, scatter_map, out2, st);
+    if (cpl <= 16) return launch_warp_bf16<16>(in, rows, n_rows, D, out, scatter_map, out2, st);
+    if (cpl <= 20) return launch_warp_bf16<20>(in, rows, n_rows, D, out, scatter_map, out2, st);
+    if (cpl <= 24) return launch_warp_bf16<24>(in, rows, n_rows, D, out, scatter_map, out2, st);
+    return launch_warp_bf16<32>(in, rows, n_rows, D, out, scatter_map, out2, st);
 }
 
 template <typename T>
@@ -181,15 +204,7 @@ void launch_t(const T *in, const int32_t *rows, int n_rows, int D, __nv_bfloat16
               cudaStream_t st) {
     const int C = D / 8;
     echo::LaunchScope ls(ECHO_K_LAYERNORM, n_rows, D, 0, st);
-    if constexpr (sizeof(T) == 2) {
-        const int cpl = (C + 31) / 32;   // 16-byte chunks per lane
-        if (cpl <= 4) return launch_warp_bf16<4>(in, rows, n_rows, D, out, st);
-        if (cpl <= 8) return launch_warp_bf16<8>(in, rows, n_rows, D, out, st);
-        if (cpl <= 16) return launch_warp_bf16<16>(in, rows, n_rows, D, out, st);
-        if (cpl <= 20) return launch_warp_bf16<20>(in, rows, n_rows, D, out, st);
-        if (cpl <= 24) return launch_warp_bf16<24>(in, rows, n_rows, D, out, st);
-        return launch_warp_bf16<32>(in, rows, n_rows, D, out, st);
-    }
+    if constexpr (sizeof(T) == 2) return launch_bf16(in, rows, n_rows, D, out, nullptr, nullptr, st);
     if (C <= 32 * kMaxChunks / 2) {   // D <= 1024: a warp per row
         constexpr int RPB = kThreads / 32;
         int grid = (n_rows + RPB - 1) / RPB;
@@ -206,6 +221,15 @@ void launch_t(const T *in, const int32_t *rows, int n_rows, int D, __nv_bfloat16
 }  // namespace
 
 namespace echo {
+
+void launch_layernorm_scatter(const void *in, int32_t n_rows, int32_t D, void *out,
+                              const int32_t *scatter_map, void *out2, cudaStream_t st) {
+    if (n_rows <= 0) return;
+    LaunchScope ls(ECHO_K_LAYERNORM, n_rows, D, 0, st);
+    launch_bf16(static_cast<const __nv_bfloat16 *>(in), nullptr, n_rows, D,
+                static_cast<__nv_bfloat16 *>(out), scatter_map, static_cast<__nv_bfloat16 *>(out2),
+                st);
+}
 
 void launch_layernorm(const void *in, echo_dtype in_t, const int32_t *rows, int32_t n_rows,
                       int32_t D, void *out, cudaStream_t st) {
