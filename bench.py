@@ -134,7 +134,8 @@ def algorithmic_work(name, m, n, k, K, xbytes=2):
     if name == "quant_scatter":
         return None, m * n * 3 + 8.0 * m
     if name == "layernorm_gather":
-        return None, m * n * 4
+        # the LN over every latent (m == NT rows) also writes the K active rows' copy
+        return None, m * n * 4 + (2.0 * K * n if m > K else 0.0)
     if name == "step_delta" and m > 0:
         return None, 2.0 * m * n
     return None, None
@@ -349,6 +350,16 @@ def job_tokens_per_s(tokens_per_replica: int, world: int, ms: float) -> float:
     return world * tokens_per_replica / (ms * 1e-3)
 
 
+def make_stack(args, w, blocks, dev):
+    """The CachedStack of the requested cache form and selection."""
+    from paper_2608_02474_gb300 import echocache as ec
+    from paper_2608_02474_gb300.pipeline import CachedStack
+    kinds = {"int8": ec.CACHE_INT8, "bf16": ec.CACHE_BF16, "ref": ec.CACHE_REF}
+    return CachedStack(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc, blocks, device=dev,
+                       cache_kind=kinds[args.cache], seg_len=args.seg_len or w.Wp, tau=args.tau,
+                       selection=args.select)
+
+
 def run_sweep(args, w, blocks, x0, xs, dev, rank, world):
     """Cached step time for every (audio profile, ratio) and the uncached block."""
     import torch
@@ -358,11 +369,7 @@ def run_sweep(args, w, blocks, x0, xs, dev, rank, world):
 
     profiles = w.sweep_profiles or (args.profile,)
     ratios = w.sweep_ratios or ((w.ratio_num, w.ratio_den),)
-    kinds = {"int8": ec.CACHE_INT8, "bf16": ec.CACHE_BF16, "ref": ec.CACHE_REF}
-    seg_len = args.seg_len or w.Wp
-    stack = CachedStack(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc, blocks, device=dev,
-                        cache_kind=kinds[args.cache], seg_len=seg_len, tau=args.tau,
-                        selection=args.select)
+    stack = make_stack(args, w, blocks, dev)
     x0_d = torch.from_numpy(x0).to(dev, torch.bfloat16)
     xs_d = [torch.from_numpy(x).to(dev, torch.bfloat16) for x in xs]
     stream = torch.cuda.current_stream()
@@ -457,7 +464,8 @@ def main():
     if args.sweep:
         run_sweep(args, w, blocks, x0, xs, dev, rank, world)
         return
-    stack = CachedStack(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc, blocks, device=dev)
+    stack = make_stack(args, w, blocks, dev)
+    seg_len = args.seg_len or w.Wp
     audio_d = torch.from_numpy(audio).to(dev)
     x0_d = torch.from_numpy(x0).to(dev, torch.bfloat16)
     xs_d = [torch.from_numpy(x).to(dev, torch.bfloat16) for x in xs]
