@@ -134,8 +134,9 @@ def algorithmic_work(name, m, n, k, K, xbytes=2):
     if name == "quant_scatter":
         return None, m * n * 3 + 8.0 * m
     if name == "layernorm_gather":
-        # the LN over every latent (m == NT rows) also writes the K active rows' copy
-        return None, m * n * 4 + (2.0 * K * n if m > K else 0.0)
+        # k = input element bytes; the LN over every latent (m > K rows) also
+        # writes the K active rows' copy
+        return None, m * n * ((k or 2) + 2.0) + (2.0 * K * n if m > K else 0.0)
     if name == "step_delta" and m > 0:
         return None, 2.0 * m * n
     return None, None

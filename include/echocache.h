@@ -446,8 +446,8 @@ echo_status echo_profile_enable(int32_t on);
  * launch's shape m, n, k as described below, and its device time in ms) into
  * the host arrays, clears the record list and returns the number copied (or
  * -1 on a CUDA error).  Shapes: GEMM (M, N, Kd); ATTENTION (M queries, L keys,
- * H * d); DRIFT (NT, D, 0); TOPK (NT, K, 0); LAYERNORM, QUANT, DEQUANT,
- * MERGE (rows, D, 0); ENERGY (T, frames, n_fft); STEP_DELTA (n, element bytes, 0)
+ * H * d); DRIFT (NT, D, 0); TOPK (NT, K, 0); LAYERNORM (rows, D, input element
+ * bytes); QUANT, DEQUANT, MERGE (rows, D, 0); ENERGY (T, frames, n_fft); STEP_DELTA (n, element bytes, 0)
  * for the reduction and (0, 0, blocks) for its final combine; UNIFORM (NT, K, 0);
  * REF_SCAN, REF_ALLOC, REF_STORE, CACHE_COPY (rows, D, 0). */
 int32_t echo_profile_read(int32_t max, int32_t *kinds, int64_t *m, int64_t *n, int64_t *k,

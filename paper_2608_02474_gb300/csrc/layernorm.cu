@@ -203,7 +203,7 @@ template <typename T>
 void launch_t(const T *in, const int32_t *rows, int n_rows, int D, __nv_bfloat16 *out,
               cudaStream_t st) {
     const int C = D / 8;
-    echo::LaunchScope ls(ECHO_K_LAYERNORM, n_rows, D, 0, st);
+    echo::LaunchScope ls(ECHO_K_LAYERNORM, n_rows, D, (int64_t)sizeof(T), st);
     if constexpr (sizeof(T) == 2) return launch_bf16(in, rows, n_rows, D, out, nullptr, nullptr, st);
     if (C <= 32 * kMaxChunks / 2) {   // D <= 1024: a warp per row
         constexpr int RPB = kThreads / 32;
@@ -225,7 +225,7 @@ namespace echo {
 void launch_layernorm_scatter(const void *in, int32_t n_rows, int32_t D, void *out,
                               const int32_t *scatter_map, void *out2, cudaStream_t st) {
     if (n_rows <= 0) return;
-    LaunchScope ls(ECHO_K_LAYERNORM, n_rows, D, 0, st);
+    LaunchScope ls(ECHO_K_LAYERNORM, n_rows, D, 2, st);
     launch_bf16(static_cast<const __nv_bfloat16 *>(in), nullptr, n_rows, D,
                 static_cast<__nv_bfloat16 *>(out), scatter_map, static_cast<__nv_bfloat16 *>(out2),
                 st);
