@@ -326,7 +326,8 @@ def run_reference(args, w, rnum, rden, rank):
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": w.name, "tokens": w.NT, "D": w.D, "heads": f"{w.H}x{w.d}",
                        "ffn": w.F, "audio_tokens": w.Lc, "ratio": f"{rnum}/{rden}",
-                       "layers": w.layers},
+                       "layers": w.layers, "cache": args.cache, "selection": args.select,
+                       "latents": args.latents},
             "cpu_baseline": {"value": round(val, 2), "unit": UNIT, "cores": cpu_cores(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": round(val, 2), "unit": UNIT, "h2d_bytes_per_step": 0,
