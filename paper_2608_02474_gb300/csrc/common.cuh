@@ -127,6 +127,15 @@ ECHO_DEV void tma_load_2d(void *dst, const CUtensorMap *m, uint64_t *bar, int32_
         : "memory");
 }
 
+// 1-D bulk copy global -> shared, completing `bytes` on `bar` (addresses
+// 16-byte aligned, bytes a multiple of 16)
+ECHO_DEV void bulk_load_1d(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+        ::"r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
+
 // ---------------------------------------------------------------------------
 // tcgen05 (5th-generation tensor cores, accumulators in tensor memory)
 // ---------------------------------------------------------------------------

@@ -176,6 +176,129 @@ layernorm_warp_bf16(const __nv_bfloat16 *__restrict__ in, const int32_t *__restr
     }
 }
 
+// All rows of a bf16 input (no gather), for D <= 8192: one warp per row as in
+// layernorm_warp_bf16, but each warp streams its rows through two shared-memory
+// buffers filled by 1-D bulk copies, the next row's copy in flight while the
+// current row is normalised and written.  Same arithmetic, same bits.
+constexpr int kBulkWarps = 4;
+
+template <int CPL>
+__global__ void __launch_bounds__(kBulkWarps * 32)
+layernorm_bulk_bf16(const __nv_bfloat16 *__restrict__ in, int n_rows, int D,
+                    __nv_bfloat16 *__restrict__ out, const int32_t *__restrict__ scatter_map,
+                    __nv_bfloat16 *__restrict__ out2, int *err) {
+    extern __shared__ __align__(128) uint8_t smem_rows[];
+    __shared__ __align__(8) uint64_t bar[kBulkWarps][2];
+    __shared__ int abort_flag;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t row_bytes = (uint32_t)D * 2u;
+    uint8_t *buf = smem_rows + (size_t)warp * 2 * row_bytes;
+    if (lane == 0) {
+        mbar_init(&bar[warp][0], 1);
+        mbar_init(&bar[warp][1], 1);
+    }
+    if (threadIdx.x == 0) abort_flag = 0;
+    fence_barrier_init();
+    __syncthreads();
+    volatile int *abort_v = &abort_flag;
+    const int C = D >> 3;
+    const float invD = 1.f / (float)D;
+    const int nw = gridDim.x * kBulkWarps;
+    int j = blockIdx.x * kBulkWarps + warp;
+    if (j < n_rows && lane == 0) {
+        mbar_arrive_expect_tx(&bar[warp][0], row_bytes);
+        bulk_load_1d(buf, in + (int64_t)j * D, row_bytes, &bar[warp][0]);
+    }
+    bool pending_next = false;
+    for (int it = 0; j < n_rows; ++it, j += nw) {
+        const int b = it & 1;
+        const int jn = j + nw;
+        __syncwarp();   // every lane is done with buffer b ^ 1 (read in the last iteration)
+        pending_next = jn < n_rows;
+        if (pending_next && lane == 0) {
+            fence_proxy_async_smem();
+            mbar_arrive_expect_tx(&bar[warp][b ^ 1], row_bytes);
+            bulk_load_1d(buf + (b ^ 1) * row_bytes, in + (int64_t)jn * D, row_bytes,
+                         &bar[warp][b ^ 1]);
+        }
+        if (!__all_sync(0xffffffffu, mbar_wait(&bar[warp][b], (it >> 1) & 1, abort_v, err))) {
+            pending_next = false;   // the CTA gives up; let the next copy land first
+            if (jn < n_rows)
+                mbar_wait(&bar[warp][b ^ 1], ((it + 1) >> 1) & 1, abort_v, nullptr, 100000000ull);
+            break;
+        }
+        const uint4 *src = reinterpret_cast<const uint4 *>(buf + b * row_bytes);
+        uint4 v[CPL];
+#pragma unroll
+        for (int k = 0; k < CPL; ++k) {
+            const int c = lane + 32 * k;
+            v[k] = c < C ? src[c] : make_uint4(0, 0, 0, 0);
+        }
+        float s = 0.f;
+#pragma unroll
+        for (int k = 0; k < CPL; ++k) {
+            float f[8];
+            unpack8_bf16(v[k], f);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) s += f[e];
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        const float mean = s * invD;
+        float ss = 0.f;
+#pragma unroll
+        for (int k = 0; k < CPL; ++k) {
+            if (lane + 32 * k < C) {
+                float f[8];
+                unpack8_bf16(v[k], f);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const float dlt = f[e] - mean;
+                    ss += dlt * dlt;
+                }
+            }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+        const float rstd = rsqrtf(ss * invD + 1e-6f);
+        uint4 *dst = reinterpret_cast<uint4 *>(out + (int64_t)j * D);
+        const int j2 = scatter_map ? scatter_map[j] : -1;
+        uint4 *dst2 = j2 >= 0 ? reinterpret_cast<uint4 *>(out2 + (int64_t)j2 * D) : nullptr;
+#pragma unroll
+        for (int k = 0; k < CPL; ++k) {
+            const int c = lane + 32 * k;
+            if (c < C) {
+                float f[8];
+                unpack8_bf16(v[k], f);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) f[e] = (f[e] - mean) * rstd;
+                const uint4 o = pack8_bf16(f);
+                dst[c] = o;
+                if (dst2) dst2[c] = o;
+            }
+        }
+    }
+    (void)pending_next;
+}
+
+template <int CPL>
+void launch_bulk_bf16(const __nv_bfloat16 *in, int n_rows, int D, __nv_bfloat16 *out,
+                      const int32_t *scatter_map, __nv_bfloat16 *out2, cudaStream_t st) {
+    const size_t smem = (size_t)kBulkWarps * 2 * D * sizeof(__nv_bfloat16);
+    static int attr_done[64] = {};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+        cudaFuncSetAttribute(layernorm_bulk_bf16<CPL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)(kBulkWarps * 2 * 8192 * sizeof(__nv_bfloat16)));
+        attr_done[dev] = 1;
+    }
+    int grid = (n_rows + kBulkWarps - 1) / kBulkWarps;
+    if (grid > 152 * 2) grid = 152 * 2;
+    layernorm_bulk_bf16<CPL><<<grid, kBulkWarps * 32, smem, st>>>(in, n_rows, D, out, scatter_map,
+                                                                  out2, echo::device_error_ptr());
+}
+
 template <int CPL>
 void launch_warp_bf16(const __nv_bfloat16 *in, const int32_t *rows, int n_rows, int D,
                       __nv_bfloat16 *out, const int32_t *scatter_map, __nv_bfloat16 *out2,
@@ -226,9 +349,13 @@ void launch_layernorm_scatter(const void *in, int32_t n_rows, int32_t D, void *o
                               const int32_t *scatter_map, void *out2, cudaStream_t st) {
     if (n_rows <= 0) return;
     LaunchScope ls(ECHO_K_LAYERNORM, n_rows, D, 2, st);
-    launch_bf16(static_cast<const __nv_bfloat16 *>(in), nullptr, n_rows, D,
-                static_cast<__nv_bfloat16 *>(out), scatter_map, static_cast<__nv_bfloat16 *>(out2),
-                st);
+    const __nv_bfloat16 *i = static_cast<const __nv_bfloat16 *>(in);
+    __nv_bfloat16 *o = static_cast<__nv_bfloat16 *>(out), *o2 = static_cast<__nv_bfloat16 *>(out2);
+    const int cpl = (D / 8 + 31) / 32;
+    if (cpl <= 16) return launch_bulk_bf16<16>(i, n_rows, D, o, scatter_map, o2, st);
+    if (cpl <= 20) return launch_bulk_bf16<20>(i, n_rows, D, o, scatter_map, o2, st);
+    if (cpl <= 24) return launch_bulk_bf16<24>(i, n_rows, D, o, scatter_map, o2, st);
+    return launch_bulk_bf16<32>(i, n_rows, D, o, scatter_map, o2, st);
 }
 
 void launch_layernorm(const void *in, echo_dtype in_t, const int32_t *rows, int32_t n_rows,
