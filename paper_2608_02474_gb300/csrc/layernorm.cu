@@ -322,12 +322,26 @@ void launch_bf16(const __nv_bfloat16 *in, const int32_t *rows, int n_rows, int D
     return launch_warp_bf16<32>(in, rows, n_rows, D, out, scatter_map, out2, st);
 }
 
+// every row of a bf16 input, optionally also scattered through a map: the
+// bulk-copy kernel (the same arithmetic as layernorm_warp_bf16)
+void launch_all_bf16(const __nv_bfloat16 *in, int n_rows, int D, __nv_bfloat16 *out,
+                     const int32_t *scatter_map, __nv_bfloat16 *out2, cudaStream_t st) {
+    const int cpl = (D / 8 + 31) / 32;
+    if (cpl <= 16) return launch_bulk_bf16<16>(in, n_rows, D, out, scatter_map, out2, st);
+    if (cpl <= 20) return launch_bulk_bf16<20>(in, n_rows, D, out, scatter_map, out2, st);
+    if (cpl <= 24) return launch_bulk_bf16<24>(in, n_rows, D, out, scatter_map, out2, st);
+    return launch_bulk_bf16<32>(in, n_rows, D, out, scatter_map, out2, st);
+}
+
 template <typename T>
 void launch_t(const T *in, const int32_t *rows, int n_rows, int D, __nv_bfloat16 *out,
               cudaStream_t st) {
     const int C = D / 8;
     echo::LaunchScope ls(ECHO_K_LAYERNORM, n_rows, D, (int64_t)sizeof(T), st);
-    if constexpr (sizeof(T) == 2) return launch_bf16(in, rows, n_rows, D, out, nullptr, nullptr, st);
+    if constexpr (sizeof(T) == 2) {
+        if (!rows) return launch_all_bf16(in, n_rows, D, out, nullptr, nullptr, st);
+        return launch_bf16(in, rows, n_rows, D, out, nullptr, nullptr, st);
+    }
     if (C <= 32 * kMaxChunks / 2) {   // D <= 1024: a warp per row
         constexpr int RPB = kThreads / 32;
         int grid = (n_rows + RPB - 1) / RPB;
@@ -349,13 +363,9 @@ void launch_layernorm_scatter(const void *in, int32_t n_rows, int32_t D, void *o
                               const int32_t *scatter_map, void *out2, cudaStream_t st) {
     if (n_rows <= 0) return;
     LaunchScope ls(ECHO_K_LAYERNORM, n_rows, D, 2, st);
-    const __nv_bfloat16 *i = static_cast<const __nv_bfloat16 *>(in);
-    __nv_bfloat16 *o = static_cast<__nv_bfloat16 *>(out), *o2 = static_cast<__nv_bfloat16 *>(out2);
-    const int cpl = (D / 8 + 31) / 32;
-    if (cpl <= 16) return launch_bulk_bf16<16>(i, n_rows, D, o, scatter_map, o2, st);
-    if (cpl <= 20) return launch_bulk_bf16<20>(i, n_rows, D, o, scatter_map, o2, st);
-    if (cpl <= 24) return launch_bulk_bf16<24>(i, n_rows, D, o, scatter_map, o2, st);
-    return launch_bulk_bf16<32>(i, n_rows, D, o, scatter_map, o2, st);
+    launch_all_bf16(static_cast<const __nv_bfloat16 *>(in), n_rows, D,
+                    static_cast<__nv_bfloat16 *>(out), scatter_map,
+                    static_cast<__nv_bfloat16 *>(out2), st);
 }
 
 void launch_layernorm(const void *in, echo_dtype in_t, const int32_t *rows, int32_t n_rows,
