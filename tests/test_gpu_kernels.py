@@ -234,6 +234,25 @@ def test_layernorm(ec, D, in_t):
     assert np.all(np.abs(g - ref) <= 2 ** -8 * np.abs(ref) + 2e-3)
 
 
+@pytest.mark.parametrize("in_t", ["bf16", "f32"])
+@pytest.mark.parametrize("n,D", [(1000, 64), (333, 1024), (1217, 5120), (90, 8192)])
+def test_layernorm_all_rows(ec, n, D, in_t):
+    """Every row (no gather): the bf16 form streams rows through shared memory
+    by bulk copies; its bits equal those of the gathered form on the same rows."""
+    x = G.random_rows(n, D, seed=D + n, scale=2.0) + F32(0.5)
+    if in_t == "bf16":
+        x = G.to_bf16_values(x)
+    src = bf(x) if in_t == "bf16" else f32(x)
+    out = ec.echo_layernorm(src)
+    ref = oracle.block.layer_norm(x)
+    g = out.float().cpu().numpy()
+    assert np.all(np.abs(g - ref) <= 2 ** -8 * np.abs(ref) + 2e-3)
+    if in_t == "bf16":
+        rows = torch.arange(n, dtype=torch.int32, device=DEV)
+        assert torch.equal(out, ec.echo_layernorm(src, rows))
+    no_device_error(ec)
+
+
 # ---------------------------------------------------------------- GEMM
 GEMM_CASES = [
     # M, Kd, N
