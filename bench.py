@@ -554,6 +554,7 @@ def main():
 
     cache_bytes = stack.cache_bytes()
     cache_bytes_rs = stack.cache_bytes(right_sized=True)
+    peak_bytes = torch.cuda.max_memory_allocated(dev)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
@@ -586,6 +587,7 @@ def main():
             line["config"]["ref_cache"] = {
                 "tau": args.tau, "seg_len": seg_len, "live_references": live,
                 "pool_high_water": hw}
+        line["peak_memory_bytes"] = peak_bytes
         line["cache_bytes"] = {"allocated": cache_bytes,
                                "right_sized": cache_bytes_rs,
                                "note": "device bytes of every layer's cache after the timed "

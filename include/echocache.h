@@ -423,6 +423,15 @@ echo_status echo_attention(const void *Q, int64_t ldq, const void *K, const void
 echo_status echo_layernorm(const void *in, echo_dtype in_t, const int32_t *rows,
                            int32_t n_rows, int32_t D, void *out, echo_stream_t stream);
 
+/* ---- failure detection (no counterpart in the paper) ---- */
+
+/* Runs the bounded-wait path every library kernel uses on one barrier that
+ * nothing completes: one thread waits limit_ns (1 us .. 2 s), gives up, sets
+ * the device flag ECHO_ERR_TIMEOUT and returns, leaving the context usable.
+ * The next echo_get_device_error reports (and clears) it.  For tests of the
+ * timeout handling.  Errors: INVALID_ARG (limit), CUDA. */
+echo_status echo_check_timeout_path(int64_t limit_ns, echo_stream_t stream);
+
 /* ---- instrumentation (no counterpart in the paper: measurement only) ---- */
 
 /* Kernel kinds reported by the profiler. */

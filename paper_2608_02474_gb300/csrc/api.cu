@@ -204,3 +204,28 @@ extern "C" echo_status echo_get_device_error(echo_stream_t stream) {
     }
     return static_cast<echo_status>(v);
 }
+
+namespace {
+
+// One thread waits for the first phase of a shared-memory barrier that no one
+// arrives at, with the library's bounded wait: after limit_ns it gives up and
+// sets ECHO_ERR_TIMEOUT, as every wait in the library does.
+__global__ void timeout_probe_kernel(uint64_t limit_ns, int *err) {
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ int abort_flag;
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_barrier_init();
+    mbar_wait(&bar, 0, &abort_flag, err, limit_ns);
+}
+
+}  // namespace
+
+extern "C" echo_status echo_check_timeout_path(int64_t limit_ns, echo_stream_t stream) {
+    using namespace echo;
+    if (limit_ns < 1000 || limit_ns > 2000000000ll) return ECHO_ERR_INVALID_ARG;
+    if (!device_supported()) return ECHO_ERR_UNSUPPORTED;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    timeout_probe_kernel<<<1, 1, 0, st>>>((uint64_t)limit_ns, device_error_ptr());
+    return last_launch_status();
+}

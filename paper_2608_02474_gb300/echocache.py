@@ -96,6 +96,7 @@ _SIGS = {
                            _i32, _vp]),
     "echo_attention": (_i32, [_vp, _i64, _vp, _vp, _i64, _i32, _i32, _i32, _i32, _vp, _i64, _vp]),
     "echo_layernorm": (_i32, [_vp, _i32, _vp, _i32, _i32, _vp, _vp]),
+    "echo_check_timeout_path": (_i32, [_i64, _vp]),
     "echo_launch_count": (_c.c_uint64, []),
     "echo_profile_enable": (_i32, [_i32]),
     "echo_profile_read": (_i32, [_i32, _vp, _vp, _vp, _vp, _vp]),
@@ -317,6 +318,10 @@ def echo_layernorm(inp, rows=None, out=None, stream=None):
     _check("echo_layernorm", lib().echo_layernorm(
         _p(inp), _dtype(inp), _p(rows), n, D, _p(out), _stream(stream)))
     return out
+
+
+def echo_check_timeout_path(limit_ns: int = 1_000_000, stream=None):
+    _check("echo_check_timeout_path", lib().echo_check_timeout_path(int(limit_ns), _stream(stream)))
 
 
 def echo_launch_count() -> int:

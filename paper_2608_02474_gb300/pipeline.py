@@ -11,6 +11,9 @@ of the step before.
 """
 from __future__ import annotations
 
+import json
+import os
+
 import torch
 
 from . import echocache as ec
@@ -98,6 +101,11 @@ class CachedStack:
         self.ws = torch.empty(ws, dtype=torch.uint8, device=dev)
         self.keys = torch.empty(self.NT, dtype=torch.float32, device=dev)
         self.gen = torch.Generator(device=dev).manual_seed(seed)
+        # ECHO_PROFILE=<path>: bracket every library launch with CUDA events;
+        # profile_report() aggregates them (and writes JSON to <path>)
+        self.profile_path = os.environ.get("ECHO_PROFILE") or None
+        if self.profile_path:
+            ec.echo_profile_enable(True)
         self.sel_ws = torch.empty(ec.echo_select_workspace_size(T, N), dtype=torch.uint8, device=dev)
         self.idx = torch.empty(self.NT, dtype=torch.int32, device=dev)
         self.all_idx = torch.arange(self.NT, dtype=torch.int32, device=dev)
@@ -151,6 +159,51 @@ class CachedStack:
             self.last_K.append(K)
             cur = dst
         return cur
+
+    # ---- checkpoint / resume of the cross-step state (the per-layer caches) ----
+    def cache_state(self) -> dict:
+        """Host copy of every layer's cache (the only state carried across steps)."""
+        if self.caches is None:
+            layers = [{"q": q.cpu(), "scale": s.cpu()} for q, s in zip(self.cache_q, self.cache_s)]
+        else:
+            layers = [{n: t.cpu() for n, t in c.t.items()} for c in self.caches]
+        return {"kind": int(self.cache_kind), "NT": self.NT, "D": self.D, "layers": layers}
+
+    def load_cache_state(self, state: dict):
+        """Restore caches saved by cache_state (same form, shapes and layer count)."""
+        if (state["kind"], state["NT"], state["D"]) != (int(self.cache_kind), self.NT, self.D):
+            raise ValueError("cache state does not match this stack")
+        if len(state["layers"]) != len(self.blocks):
+            raise ValueError("cache state has a different number of layers")
+        for l, layer in enumerate(state["layers"]):
+            if self.caches is None:
+                self.cache_q[l].copy_(layer["q"])
+                self.cache_s[l].copy_(layer["scale"])
+            else:
+                for n, t in self.caches[l].t.items():
+                    t.copy_(layer[n])
+
+    def save_caches(self, path: str):
+        torch.save(self.cache_state(), path)
+
+    def load_caches(self, path: str):
+        self.load_cache_state(torch.load(path))
+
+    def profile_report(self) -> dict:
+        """Per-kernel totals of the launches recorded since the last report
+        (profiling is on when ECHO_PROFILE is set); written as JSON to the
+        ECHO_PROFILE path."""
+        agg = {}
+        for name, m, n, k, ms in ec.echo_profile_read():
+            a = agg.setdefault(f"{name}[{m}x{n}x{k}]", {"launches": 0, "ms": 0.0})
+            a["launches"] += 1
+            a["ms"] += ms
+        for a in agg.values():
+            a["ms_per_launch"] = a["ms"] / a["launches"]
+        if self.profile_path:
+            with open(self.profile_path, "w") as f:
+                json.dump(agg, f, indent=1)
+        return agg
 
     def cache_bytes(self, right_sized: bool = False) -> int:
         """Device bytes of every layer's cache; with right_sized, a reference

@@ -201,3 +201,9 @@ def test_cache_form_argument_checks(ec):
     assert L.echo_block_step_cache(ctypes.byref(w), ctypes.byref(dims), _vp(FAKE), _vp(FAKE), 4,
                                    ctypes.byref(mk(NT=65)), _vp(FAKE), _vp(FAKE), 1 << 30,
                                    None) == 2
+
+
+def test_timeout_probe_argument_checks(ec):
+    L = ec.lib()
+    assert L.echo_check_timeout_path(999, None) == 1
+    assert L.echo_check_timeout_path(3_000_000_000, None) == 1
