@@ -4,7 +4,7 @@
 // P_k = c_k |X_k|^2 / n_fft is summed over the segment's frames per bin and then
 // per linear band; energy = sqrt(sum of the bands).
 //
-// One CTA per segment, four frame groups of 256 threads.  Each thread keeps
+// One CTA per segment, eight frame groups of 128 threads.  Each thread keeps
 // the frame-summed power of its bins in registers, so the result does not
 // depend on scheduling: groups are combined in a fixed order and bands are
 // reduced by warps in a fixed order.
@@ -13,9 +13,9 @@
 
 namespace {
 
-constexpr int kGroup = 256;          // threads per frame group
-constexpr int kGroups = 4;           // frame groups per CTA
-constexpr int kMaxBinsPerThread = 9; // (4096/2 + 1) / 256 rounded up
+constexpr int kGroup = 128;           // threads per frame group
+constexpr int kGroups = 8;            // frame groups per CTA
+constexpr int kMaxBinsPerThread = 17; // (4096/2 + 1) / 128 rounded up
 
 __global__ void __launch_bounds__(kGroup *kGroups)
 segment_energy_kernel(const float *__restrict__ audio, int seg_len, int n_fft, int log2n, int hop,
