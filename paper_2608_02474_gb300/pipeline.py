@@ -111,15 +111,49 @@ class CachedStack:
         self.all_idx = torch.arange(self.NT, dtype=torch.int32, device=dev)
         self.scores = torch.empty(self.NT, dtype=torch.float32, device=dev)
         self.y = [torch.empty(self.NT, D, dtype=torch.bfloat16, device=dev) for _ in range(2)]
-        self.band = torch.empty(T, 8, dtype=torch.float32, device=dev)
-        self.seg = torch.zeros(T, dtype=torch.float32, device=dev)
+        # The audio energy runs on a side stream into two alternating buffers:
+        # it depends on the audio only, so a step's energy is computed while
+        # the previous step's kernels still run; the step waits for it before
+        # its first selection.
+        self._aud_stream = torch.cuda.Stream(dev)
+        self._band = [torch.empty(T, 8, dtype=torch.float32, device=dev) for _ in range(2)]
+        self._seg = [torch.zeros(T, dtype=torch.float32, device=dev) for _ in range(2)]
+        self._seg_ready = [torch.cuda.Event() for _ in range(2)]
+        self._seg_free = [torch.cuda.Event() for _ in range(2)]
+        self._next_buf, self._pending, self._in_use = 0, None, 0
+        self._audio_key = None
+        self.band, self.seg = self._band[0], self._seg[0]
         self.last_K = []
 
     def set_audio(self, audio: torch.Tensor, n_fft: int = 512, hop: int = 160, n_bands: int = 8):
-        if self.band.shape[1] != n_bands:
-            self.band = torch.empty(self.T, n_bands, dtype=torch.float32, device=self.seg.device)
-        ec.echo_audio_energy(audio, self.T, n_fft, hop, n_bands, self.band, self.seg)
+        """Segment energy of the audio (Sec. 3.3) for the next step.  The result
+        is written on a side stream; the next step waits for it, and a caller
+        that reads the returned tensors directly calls wait_audio() first."""
+        dev = self.seg.device
+        main = torch.cuda.current_stream(dev)
+        side = self._aud_stream
+        b = self._next_buf
+        self._next_buf ^= 1
+        if self._band[b].shape[1] != n_bands:
+            self._band[b] = torch.empty(self.T, n_bands, dtype=torch.float32, device=dev)
+        side.wait_event(self._seg_free[b])          # the last step that read buffer b is done
+        key = (audio.data_ptr(), audio._version)
+        if key != self._audio_key:                  # new audio: order after its writes
+            ev = torch.cuda.Event()
+            ev.record(main)
+            side.wait_event(ev)
+            self._audio_key = key
+        ec.echo_audio_energy(audio, self.T, n_fft, hop, n_bands, self._band[b], self._seg[b],
+                             stream=side)
+        self._seg_ready[b].record(side)
+        self._pending = b
+        self.band, self.seg = self._band[b], self._seg[b]
         return self.band, self.seg
+
+    def wait_audio(self):
+        """Make the current stream wait for the last set_audio's result."""
+        if self._pending is not None:
+            torch.cuda.current_stream(self.seg.device).wait_event(self._seg_ready[self._pending])
 
     def step(self, x: torch.Tensor, ratio_num: int, ratio_den: int, full: bool = False,
              keep_scores: bool = False, out: torch.Tensor | None = None) -> torch.Tensor:
@@ -128,6 +162,10 @@ class CachedStack:
         cur = x
         self.last_K = []
         last = len(self.blocks) - 1
+        main = torch.cuda.current_stream(self.seg.device)
+        if self._pending is not None:               # this step uses the newest energy
+            main.wait_event(self._seg_ready[self._pending])
+            self._in_use, self._pending = self._pending, None
         for l, blk in enumerate(self.blocks):
             if full:
                 idx, K = self.all_idx, self.NT
@@ -158,6 +196,7 @@ class CachedStack:
                                          workspace=self.ws)
             self.last_K.append(K)
             cur = dst
+        self._seg_free[self._in_use].record(main)   # set_audio may now overwrite it
         return cur
 
     # ---- checkpoint / resume of the cross-step state (the per-layer caches) ----
