@@ -185,3 +185,52 @@ def test_layer_step_with_cache_forms_teacher_forced(ec, kind):
         for n in g.t:
             assert torch.equal(g.t[n], before.t[n]), n
         o = res.cache
+
+
+@pytest.mark.slow
+def test_ref_cache_block_full_size_sampled(ec):
+    """The 32760-token block (D 5120, 40 heads, r = 1/5) with the reference
+    cache (tau 0.9, segments of 52 tokens) on spatially smooth latents: the
+    oracle's cache state is loaded, indices and inactive rows are bit-exact,
+    64 sampled active rows are held to the normwise bars, and the cache write
+    equals echo_cache_write of the rows the step returned."""
+    from synth import WAN_BLOCK_32760 as w
+    from test_gpu_block import rel_err
+    audio = G.audio(w)
+    _, e = oracle.energy.audio_energy(audio, w.T)
+    e32 = e.astype(F32)
+    W, cond = G.block_weights(w, 0), G.cond_tokens(w, audio)
+    x0 = G.latents_smooth(w)
+    x1 = G.step_input(w, x0, 1)
+    o = R.RefCache(w.NT, w.D, w.NT, w.Wp, 0.9)
+    o.write(np.arange(w.NT), x0)
+    live, hw = o.stats()
+    assert 0 < live < w.NT
+    g = _device_cache_from(ec, o, w)
+    before = g.clone()
+    blk = ec.DeviceBlock.from_host(W, cond)
+    dims = ec.BlockDims(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc)
+    xd = _bf(x1)
+    idx, K, _ = ec.echo_select_cache(xd, g, torch.from_numpy(e32).to(DEV), w.T, w.N, 1, 5)
+    y = ec.echo_block_step_cache(blk, dims, xd, idx, K, g)
+    torch.cuda.synchronize()
+    assert ec.echo_get_device_error() == 0
+    sc = oracle.select.scores_from(x1, o.reconstruct_f32(), e32, w.T, w.N)
+    oidx = oracle.select.top_k(sc, K)
+    gi = idx.cpu().numpy()
+    assert np.array_equal(gi, oidx)
+    gy = y.float().cpu().numpy()
+    inactive = np.setdiff1d(np.arange(w.NT), gi)
+    assert np.array_equal(gy[inactive], o.reconstruct_bf16()[inactive])
+    rng = np.random.default_rng(0)
+    top = oidx[np.argsort(-sc[oidx], kind="stable")[:32]]
+    rows = np.unique(np.concatenate([rng.choice(oidx, 32, replace=False), top]))
+    Kv, Vv = oracle.block.self_kv(x1, W)
+    Kc, Vc = oracle.block.cross_kv(cond, W)
+    ya = oracle.block.active_rows(x1, rows, W, w.H, Kv, Vv, Kc, Vc)
+    mx, mean = rel_err(gy[rows], ya)
+    assert mx <= 2e-2 and mean <= 5e-3, (mx, mean)
+    before.write(y[idx.long()].contiguous(), idx)
+    torch.cuda.synchronize()
+    for n in g.t:
+        assert torch.equal(g.t[n], before.t[n]), n
