@@ -292,6 +292,23 @@ def cpu_cores():
         return os.cpu_count()
 
 
+def cpu_model():
+    """The host CPU's model line from /proc/cpuinfo (or the machine type)."""
+    import platform
+    parts = {"0xd4f": "Neoverse-V2", "0xd40": "Neoverse-V1", "0xd0c": "Neoverse-N1"}
+    try:
+        for line in open("/proc/cpuinfo"):
+            k = line.split(":")[0].strip().lower()
+            if k in ("model name", "cpu model", "hardware"):
+                return line.split(":", 1)[1].strip()
+            if k == "cpu part":
+                v = line.split(":", 1)[1].strip().lower()
+                return f"{platform.machine()} {parts.get(v, 'part ' + v)}"
+    except OSError:
+        pass
+    return platform.machine()
+
+
 # ---------------------------------------------------------------------------
 def build_inputs(w, profile, latents="iid"):
     import numpy as np
@@ -329,6 +346,7 @@ def run_reference(args, w, rnum, rden, rank):
                        "layers": w.layers, "cache": args.cache, "selection": args.select,
                        "latents": args.latents},
             "cpu_baseline": {"value": round(val, 2), "unit": UNIT, "cores": cpu_cores(),
+                             "cpu_model": cpu_model(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": round(val, 2), "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
@@ -565,6 +583,7 @@ def main():
                                           selection=args.select, tau=args.tau,
                                           seg_len=args.seg_len or None)
         cpu = {"value": round(w.NT / step_s, 2), "unit": UNIT, "cores": cpu_cores(),
+               "cpu_model": cpu_model(),
                "kind": "oracle", "sample": sample, "ms_per_step": round(step_s * 1e3, 1)}
 
     if rank == 0:

@@ -151,14 +151,20 @@ def test_edge_ratios_and_aliasing(ec):
 
 
 @pytest.mark.slow
-@pytest.mark.parametrize("name,layer", [("wan_block_32760", 0), ("wan_stack40_32760", 39),
-                                        ("wan_sweep_63960", 0)])
-def test_wan_block_sampled_rows(ec, name, layer):
+@pytest.mark.parametrize("name,layer,step", [("wan_block_32760", 0, 1),
+                                             ("wan_stack40_32760", 39, 1),
+                                             ("wan_stack40_32760", 19, 10),
+                                             ("wan_stack40_32760", 0, 19),
+                                             ("wan_sweep_63960", 0, 1)])
+def test_wan_block_sampled_rows(ec, name, layer, step):
     """Full-size Wan2.2-S2V-shaped blocks (D 5120, 40 heads) at r = 1/5: the
-    32760-token block, the last layer of the 40-layer stack (its own weights),
-    and the 63960-token sweep shape.  Indices bit-exact, inactive rows
-    bit-exact, 64 sampled active rows (32 random, 32 of highest score) against
-    the oracle with keys/values over all tokens."""
+    32760-token block, layers 0, 19 and 39 of the 40-layer stack (each with its
+    own weights) at steps 1, 10 and 19, and the 63960-token sweep shape.  Each
+    case is teacher-forced: the layer input is the step-t input and the cache
+    holds the quantised step-(t-1) input, as if that had been the previous
+    output.  Indices bit-exact, inactive rows bit-exact, 64 sampled active rows
+    (32 random, 32 of highest score) against the oracle with keys/values over
+    all tokens."""
     from synth import ALL
     w = ALL[name]
     audio = G.audio(w)
@@ -167,8 +173,9 @@ def test_wan_block_sampled_rows(ec, name, layer):
     W = G.block_weights(w, layer)
     cond = G.cond_tokens(w, audio)
     x0 = G.latents(w)
-    x1 = G.step_input(w, x0, 1)
-    q, s, _ = oracle.cache.quantize_rows(x0)      # cache as if the previous output were x0
+    prev = x0 if step == 1 else G.step_input(w, x0, step - 1)
+    x1 = G.step_input(w, x0, step)
+    q, s, _ = oracle.cache.quantize_rows(prev)    # cache as if the previous output were prev
     blk = ec.DeviceBlock.from_host(W, cond)
     g_idx, y, qd, sd = gpu_layer(ec, blk, w, x1, q, s, e32, (w.ratio_num, w.ratio_den))
 
