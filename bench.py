@@ -520,8 +520,11 @@ def main():
     torch.cuda.synchronize()
     l0 = ec.echo_launch_count()
     ev0.record(stream)
+    host_s = 0.0
     for i in range(args.steps):
+        h0 = time.perf_counter()
         one_step(xs_d[i % 2])
+        host_s += time.perf_counter() - h0
     ev1.record(stream)
     torch.cuda.synchronize()
     barrier()
@@ -569,6 +572,8 @@ def main():
         e2e = {"value": round(job_tokens_per_s(w.NT, world, ems), 2), "unit": UNIT,
                "h2d_bytes_per_step": xh[0].numel() * 2, "d2h_bytes_per_step": yh[0].numel() * 2,
                "ms_per_step": round(ems, 3)}
+        if rate is not None:   # the budgets this leg ran (the rate state carries on)
+            e2e["budgets"] = rate.budgets[-args.steps:]
 
     cache_bytes = stack.cache_bytes()
     cache_bytes_rs = stack.cache_bytes(right_sized=True)
@@ -600,7 +605,8 @@ def main():
                            "latents": args.latents,
                            "l2": "inputs larger than L2 (x 335 MB, weights 702 MB per block)"},
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
-                "gpu_launches": launches, "kernels": table}
+                "gpu_launches": launches, "kernels": table,
+                "host_ms_per_step": round(1e3 * host_s / args.steps, 3)}
         if args.cache == "ref":
             live, hw = stack.caches[-1].stats()
             line["config"]["ref_cache"] = {
