@@ -159,13 +159,18 @@ class CachedStack:
              keep_scores: bool = False, out: torch.Tensor | None = None) -> torch.Tensor:
         """One denoising step over every layer; returns the last layer's output
         (written into `out` when given)."""
-        cur = x
-        self.last_K = []
-        last = len(self.blocks) - 1
         main = torch.cuda.current_stream(self.seg.device)
         if self._pending is not None:               # this step uses the newest energy
             main.wait_event(self._seg_ready[self._pending])
             self._in_use, self._pending = self._pending, None
+        cur = self._layers(x, ratio_num, ratio_den, full, keep_scores, out)
+        self._seg_free[self._in_use].record(main)   # set_audio may now overwrite it
+        return cur
+
+    def _layers(self, x, ratio_num, ratio_den, full, keep_scores, out):
+        cur = x
+        self.last_K = []
+        last = len(self.blocks) - 1
         for l, blk in enumerate(self.blocks):
             if full:
                 idx, K = self.all_idx, self.NT
@@ -196,8 +201,33 @@ class CachedStack:
                                          workspace=self.ws)
             self.last_K.append(K)
             cur = dst
-        self._seg_free[self._in_use].record(main)   # set_audio may now overwrite it
         return cur
+
+    def capture_step(self, x: torch.Tensor, ratio_num: int, ratio_den: int,
+                     out: torch.Tensor | None = None, audio: torch.Tensor | None = None,
+                     n_fft: int = 512, hop: int = 160, n_bands: int = 8):
+        """Record one cached step over every layer as a CUDA graph and return
+        (graph, output tensor).  graph.replay() re-runs the step on the same
+        buffers with one launch from the host: copy each step's input into `x`
+        first.  With `audio` the graph starts with the audio energy (on the
+        graph's own stream); without it, it reads the energy of the last
+        set_audio.  Selection "random" draws keys from a host generator and
+        cannot be captured.  Run one eager step of the same ratio first, so
+        that every kernel's one-time set-up is done."""
+        if self.selection == "random":
+            raise ValueError("random selection cannot be captured")
+        dev = self.seg.device
+        self.wait_audio()
+        if self._pending is not None:
+            self._in_use, self._pending = self._pending, None
+        band, seg = self._band[self._in_use], self._seg[self._in_use]
+        torch.cuda.synchronize(dev)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            if audio is not None:
+                ec.echo_audio_energy(audio, self.T, n_fft, hop, n_bands, band, seg)
+            y = self._layers(x, ratio_num, ratio_den, False, False, out)
+        return g, y
 
     # ---- checkpoint / resume of the cross-step state (the per-layer caches) ----
     def cache_state(self) -> dict:

@@ -85,3 +85,41 @@ def test_profile_report_from_env(ec, tmp_path, monkeypatch):
     assert {"gemm_tcgen05", "attention", "drift_score", "topk_select", "dequant_merge"} <= names
     assert json.loads(out.read_text()) == json.loads(json.dumps(rep))
     assert all(v["launches"] > 0 and v["ms"] >= 0 for v in rep.values())
+
+
+@pytest.mark.parametrize("kind,selection", [(0, "energy"), (2, "energy"), (0, "uniform")])
+def test_graph_replay_matches_eager_steps(ec, kind, selection):
+    """A cached step captured as a CUDA graph and replayed on new inputs gives
+    the same outputs and caches, bit for bit, as the same steps run eagerly."""
+    from paper_2608_02474_gb300.pipeline import CachedStack
+    from synth import STACK4_7800 as w
+    audio = torch.from_numpy(G.audio(w)).to(DEV)
+    cond = G.cond_tokens(w, G.audio(w))
+    blks = [ec.DeviceBlock.from_host(G.block_weights(w, l), cond) for l in range(w.layers)]
+    x0 = G.latents(w)
+    xs = [torch.from_numpy(G.step_input(w, x0, t)).to(DEV, torch.bfloat16) for t in range(1, 6)]
+    x0d = torch.from_numpy(x0).to(DEV, torch.bfloat16)
+    stacks = []
+    for _ in range(2):
+        st = CachedStack(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc, blks, cache_kind=kind, seg_len=w.Wp,
+                         tau=0.5, selection=selection)
+        st.set_audio(audio)
+        st.step(x0d, 1, 1, full=True)
+        st.step(xs[0], 1, 5)
+        stacks.append(st)
+    a, b = stacks
+    xbuf = torch.empty_like(xs[0])
+    ybuf = torch.empty_like(xs[0])
+    g, y = a.capture_step(xbuf, 1, 5, out=ybuf)
+    assert y.data_ptr() == ybuf.data_ptr()
+    for x in xs[1:]:
+        xbuf.copy_(x)
+        g.replay()
+        yb = b.step(x, 1, 5)
+        torch.cuda.synchronize()
+        assert torch.equal(ybuf, yb)
+    ca, cb = a.cache_state(), b.cache_state()
+    for la, lb in zip(ca["layers"], cb["layers"]):
+        for n in la:
+            assert torch.equal(la[n], lb[n]), n
+    assert ec.echo_get_device_error() == 0
