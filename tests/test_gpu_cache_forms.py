@@ -234,3 +234,27 @@ def test_ref_cache_block_full_size_sampled(ec):
     torch.cuda.synchronize()
     for n in g.t:
         assert torch.equal(g.t[n], before.t[n]), n
+
+
+@pytest.mark.parametrize("kind", ["bf16", "ref"])
+def test_layer_step_with_no_active_rows(ec, kind):
+    """K = 0: the step returns the cache's reconstruction and leaves the cache
+    as it was."""
+    w = TINY_256
+    W, cond = G.block_weights(w, 0), G.cond_tokens(w, G.audio(w))
+    blk = ec.DeviceBlock.from_host(W, cond)
+    dims = ec.BlockDims(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc)
+    v = G.correlated_rows(w.NT, w.D, seed=12, rho=0.9)
+    if kind == "bf16":
+        g = ec.DeviceCache(ec.CACHE_BF16, w.NT, w.D)
+    else:
+        g = ec.DeviceCache(ec.CACHE_REF, w.NT, w.D, seg_len=8, tau=0.8)
+    g.write(_bf(v), _rows(np.arange(w.NT)))
+    before = g.clone()
+    x = _bf(G.latents(w))
+    y = ec.echo_block_step_cache(blk, dims, x, None, 0, g)
+    torch.cuda.synchronize()
+    assert ec.echo_get_device_error() == 0
+    assert torch.equal(y, g.read())
+    for n in g.t:
+        assert torch.equal(g.t[n], before.t[n]), n
