@@ -132,8 +132,10 @@ def algorithmic_work(name, m, n, k, K, xbytes=2):
     if name == "drift_score":
         return None, m * n * (xbytes + 1) + 8.0 * m
     if name == "dequant_merge":
+        # inactive rows: codes and scale in, bf16 out; the active rows are
+        # already in y (stored by the FFN-down epilogue); the row map once
         NT, D = m, n
-        return None, (NT - K) * (D + 4) + K * 2 * D + NT * 2 * D + 4 * NT
+        return None, (NT - K) * (3.0 * D + 4) + 4.0 * NT
     if name == "quant_scatter":
         return None, m * n * 3 + 8.0 * m
     if name == "layernorm_gather":

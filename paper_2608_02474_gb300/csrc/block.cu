@@ -13,10 +13,11 @@
 //   attention   att = MHA(Qc, Kc, Vc)
 //   GEMM        h2 = att Woc^T + boc + h1               (fp32)
 //   LN, GEMM    u = GELU(LN(h2) W1^T + b1)
-//   GEMM        y_act = u W2^T + b2 + h2                (bf16; the epilogue
-//               also folds max |y_act| per row for the quantiser)
-//   quant       cache[idx] = Q(y_act)                   (one pass over y_act)
-//   merge       y = fresh rows at idx, reconstructed cache elsewhere
+//   GEMM        y[idx] = u W2^T + b2 + h2               (bf16, stored at the
+//               active tokens' rows of y; the epilogue also folds max |y| per
+//               row for the quantiser)
+//   merge       y = reconstructed cache at every other row
+//   quant       cache[idx] = Q(y[idx])                  (one pass)
 #include "common.cuh"
 #include "internal.h"
 
@@ -92,10 +93,11 @@ echo_status check_block(const echo_block_weights *w, const echo_block_dims *dims
     return ECHO_OK;
 }
 
-// rowmap and the block on the K active rows: y_act (bf16 [K, D]) at ws + L.yact
+// rowmap and the block on the K active rows: y_act (bf16 [K, D]) at ws + L.yact,
+// or, with y_scatter, straight into rows idx[j] of y_scatter
 echo_status run_active(const echo_block_weights *w, const echo_block_dims &d, const void *x,
                        const int32_t *idx, int32_t K, uint8_t *ws, const Layout &L,
-                       cudaStream_t st) {
+                       cudaStream_t st, void *y_scatter = nullptr) {
     using namespace echo;
     const int NT = d.T * d.N;
     int32_t *rowmap = reinterpret_cast<int32_t *>(ws + L.rowmap);
@@ -136,9 +138,10 @@ echo_status run_active(const echo_block_weights *w, const echo_block_dims &d, co
         uint32_t *amax = reinterpret_cast<uint32_t *>(ws + L.amax);
         if (cudaMemsetAsync(amax, 0, sizeof(uint32_t) * (size_t)K, st) != cudaSuccess)
             return ECHO_ERR_CUDA;
-        LinearArgs down{u, d.F, K, d.F, w->W2, w->b2, D, 0, h2, ECHO_F32, nullptr, yact, D,
-                        ECHO_BF16};
+        LinearArgs down{u, d.F, K, d.F, w->W2, w->b2, D, 0, h2, ECHO_F32, nullptr,
+                        y_scatter ? y_scatter : yact, D, ECHO_BF16};
         down.row_amax = amax;
+        if (y_scatter) down.out_rows = idx;
         s = launch_linear(down, st);
         if (s != ECHO_OK) return s;
     }
@@ -163,15 +166,17 @@ extern "C" echo_status echo_block_step(const echo_block_weights *w, const echo_b
     if (!device_supported()) return ECHO_ERR_UNSUPPORTED;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     uint8_t *ws = static_cast<uint8_t *>(workspace);
-    s = run_active(w, d, x, idx, K, ws, L, st);
+    // the FFN-down epilogue stores the active rows at their token positions in
+    // y (every read of x is done by then, so y may alias x)
+    s = run_active(w, d, x, idx, K, ws, L, st, y);
     if (s != ECHO_OK) return s;
     const int32_t *rowmap = reinterpret_cast<const int32_t *>(ws + L.rowmap);
-    // the merge reads the cache of the inactive rows only, the quantiser writes
-    // the active rows only: their order does not matter
-    launch_dequant_merge(cache_q, cache_scale, rowmap, ws + L.yact, NT, d.D, y, st);
+    // the merge fills the inactive rows from the cache; the quantiser reads the
+    // active rows of y and writes the active rows of the cache: no overlap
+    launch_dequant_merge(cache_q, cache_scale, rowmap, nullptr, NT, d.D, y, st);
     if (K > 0)
-        launch_quant_amax(ws + L.yact, reinterpret_cast<const uint32_t *>(ws + L.amax), idx, K,
-                          d.D, cache_q, cache_scale, st);
+        launch_quant_amax(y, reinterpret_cast<const uint32_t *>(ws + L.amax), idx, K, d.D,
+                          cache_q, cache_scale, st);
     return last_launch_status();
 }
 

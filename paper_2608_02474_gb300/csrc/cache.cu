@@ -98,10 +98,10 @@ quant_amax_kernel(const __nv_bfloat16 *__restrict__ src, const uint32_t *__restr
     const int warps = blockDim.x >> 5;
     const int C = D >> 3;
     for (int j = blockIdx.x * warps + (threadIdx.x >> 5); j < n_rows; j += gridDim.x * warps) {
-        const __nv_bfloat16 *s = src + (int64_t)j * D;
+        const int r = rows ? rows[j] : j;
+        const __nv_bfloat16 *s = src + (int64_t)r * D;   // the rows sit at their token positions
         const uint32_t ab = amax_bits[j];
         const float amax = __uint_as_float(ab);
-        const int r = rows ? rows[j] : j;
         int8_t *qr = q + (int64_t)r * D;
         if (ab >= 0x7F800000u) {   // NaN or infinity in the row
             for (int c = lane; c < C; c += 32) *reinterpret_cast<uint2 *>(qr + 8 * c) = make_uint2(0, 0);
@@ -178,7 +178,8 @@ __global__ void rowmap_kernel(const int32_t *__restrict__ idx, int K, int32_t *_
     if (j < K) rowmap[idx[j]] = j;
 }
 
-// y[i] = y_act[rowmap[i]] if rowmap[i] >= 0 else bf16(q[i] * s[i])
+// y[i] = y_act[rowmap[i]] if rowmap[i] >= 0 else bf16(q[i] * s[i]); without
+// y_act the active rows of y are already in place and are left alone
 __global__ void __launch_bounds__(kVecThreads)
 dequant_merge_kernel(const int8_t *__restrict__ q, const float *__restrict__ scale,
                      const int32_t *__restrict__ rowmap, const __nv_bfloat16 *__restrict__ y_act,
@@ -191,10 +192,12 @@ dequant_merge_kernel(const int8_t *__restrict__ q, const float *__restrict__ sca
         const int pos = rowmap[i];
         uint4 *o = reinterpret_cast<uint4 *>(y + (int64_t)i * D + 16 * c);
         if (pos >= 0) {
-            const uint4 *a = reinterpret_cast<const uint4 *>(y_act + (int64_t)pos * D + 16 * c);
-            const uint4 v0 = __ldcs(a), v1 = __ldcs(a + 1);
-            __stcs(o, v0);
-            __stcs(o + 1, v1);
+            if (y_act) {
+                const uint4 *a = reinterpret_cast<const uint4 *>(y_act + (int64_t)pos * D + 16 * c);
+                const uint4 v0 = __ldcs(a), v1 = __ldcs(a + 1);
+                __stcs(o, v0);
+                __stcs(o + 1, v1);
+            }
         } else {
             const int4 qv = __ldcs(reinterpret_cast<const int4 *>(q + (int64_t)i * D + 16 * c));
             float f[16];

@@ -41,6 +41,7 @@ struct GemmParams {
     const int32_t *resid_rows;
     void *out;
     int64_t ldo;
+    const int32_t *out_rows;   // output row m goes to row out_rows[m] (NULL: m)
     uint32_t *row_amax;
     int *err;
 };
@@ -176,6 +177,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
             const bool row_ok = row < p.M;
             int rrow = row;
             if ((EPI & EPI_RES_BF16) && p.resid_rows && row_ok) rrow = p.resid_rows[row];
+            const int64_t orow = (p.out_rows && row_ok) ? p.out_rows[row] : row;
             uint32_t rmax = 0;   // EPI_ROWAMAX: max |v| of this row's stored values, as bits
             for (int c = 0; c < BN; c += 32) {
                 const int col = n0 + c;
@@ -221,13 +223,13 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                 }
                 if (EPI & EPI_OUT_F32) {
                     float4 *op = reinterpret_cast<float4 *>(static_cast<float *>(p.out) +
-                                                            (int64_t)row * p.ldo + col);
+                                                            orow * p.ldo + col);
 #pragma unroll
                     for (int i = 0; i < 8; ++i)
                         op[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
                 } else {
                     uint4 *op = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.out) +
-                                                          (int64_t)row * p.ldo + col);
+                                                          orow * p.ldo + col);
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {
                         const uint4 pk = pack8_bf16(v + 8 * i);
@@ -301,6 +303,7 @@ echo_status launch_linear(const LinearArgs &a, cudaStream_t st) {
     p.resid_rows = a.resid_rows;
     p.out = a.out;
     p.ldo = a.ldo;
+    p.out_rows = a.out_rows;
     p.row_amax = a.row_amax;
     p.err = device_error_ptr();
     int epi = 0;

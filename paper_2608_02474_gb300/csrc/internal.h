@@ -54,6 +54,7 @@ struct LinearArgs {
     const void *resid; echo_dtype resid_t; const int32_t *resid_rows;
     void *out; int64_t ldo; echo_dtype out_t;
     uint32_t *row_amax = nullptr;   // bf16 out with an fp32 residual only: max |out| per row
+    const int32_t *out_rows = nullptr;   // output row m is stored at row out_rows[m]
 };
 echo_status launch_linear(const LinearArgs &a, cudaStream_t st);
 
@@ -65,7 +66,8 @@ echo_status launch_attention(const void *Q, int64_t ldq, const void *K, const vo
 // cache.cu
 void launch_quant(const void *src, echo_dtype st_t, const int32_t *rows, int32_t n_rows,
                   int32_t D, int8_t *q, float *scale, cudaStream_t st);
-// int8 quantisation of bf16 rows whose max |v| is already known (fp32 bits)
+// int8 quantisation of bf16 rows whose max |v| is already known (fp32 bits):
+// row j is read from src row rows[j] and written to cache row rows[j]
 void launch_quant_amax(const void *src, const uint32_t *amax, const int32_t *rows, int32_t n_rows,
                        int32_t D, int8_t *q, float *scale, cudaStream_t st);
 void launch_dequant(const int8_t *q, const float *scale, const int32_t *rows, int32_t n_rows,
