@@ -592,16 +592,21 @@ def main():
         barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
+        h0 = time.perf_counter()
         stack.run_host([xh[i % 2] for i in range(args.steps)],
                        [yh[i % 2] for i in range(args.steps)], rnum, rden, audio=audio_d,
                        rate=rate)
+        host_enqueue_ms = (time.perf_counter() - h0) * 1e3 / args.steps
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
         ems = slowest_rank_ms(e0.elapsed_time(e1) / args.steps, world, dev)
         e2e = {"value": round(job_tokens_per_s(w.NT, world, ems), 2), "unit": UNIT,
                "h2d_bytes_per_step": xh[0].numel() * 2, "d2h_bytes_per_step": yh[0].numel() * 2,
-               "ms_per_step": round(ems, 3)}
+               "ms_per_step": round(ems, 3),
+               # host time to enqueue a step with its copies: near the step time
+               # only where pinned copies block the host
+               "host_ms_per_step": round(host_enqueue_ms, 3)}
         if rate is not None:   # the budgets this leg ran (the rate state carries on)
             e2e["budgets"] = rate.budgets[-args.steps:]
 
