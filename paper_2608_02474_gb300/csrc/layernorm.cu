@@ -109,14 +109,10 @@ layernorm_kernel(const T *__restrict__ in, const int32_t *__restrict__ rows, int
 // bf16 input: one warp per row, the row held packed in registers (CPL 16-byte
 // chunks per lane), so each row is read from HBM once and no block barrier is
 // needed.
-// With scatter_map, row j is also written to out2[scatter_map[j]] when that is
-// >= 0: the LN of every latent (for K and V) then also yields the gathered LN
-// of the active ones (for Q') without reading them a second time.
 template <int CPL>
 __global__ void __launch_bounds__(kThreads)
 layernorm_warp_bf16(const __nv_bfloat16 *__restrict__ in, const int32_t *__restrict__ rows,
-                    int n_rows, int D, __nv_bfloat16 *__restrict__ out,
-                    const int32_t *__restrict__ scatter_map, __nv_bfloat16 *__restrict__ out2) {
+                    int n_rows, int D, __nv_bfloat16 *__restrict__ out) {
     const int lane = threadIdx.x & 31;
     const int warps = kThreads / 32;
     const int C = D >> 3;
@@ -158,8 +154,6 @@ layernorm_warp_bf16(const __nv_bfloat16 *__restrict__ in, const int32_t *__restr
         for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
         const float rstd = rsqrtf(ss * invD + 1e-6f);
         uint4 *dst = reinterpret_cast<uint4 *>(out + (int64_t)j * D);
-        const int j2 = scatter_map ? scatter_map[j] : -1;
-        uint4 *dst2 = j2 >= 0 ? reinterpret_cast<uint4 *>(out2 + (int64_t)j2 * D) : nullptr;
 #pragma unroll
         for (int k = 0; k < CPL; ++k) {
             const int c = lane + 32 * k;
@@ -168,9 +162,7 @@ layernorm_warp_bf16(const __nv_bfloat16 *__restrict__ in, const int32_t *__restr
                 unpack8_bf16(v[k], f);
 #pragma unroll
                 for (int e = 0; e < 8; ++e) f[e] = (f[e] - mean) * rstd;
-                const uint4 o = pack8_bf16(f);
-                dst[c] = o;
-                if (dst2) dst2[c] = o;
+                dst[c] = pack8_bf16(f);
             }
         }
     }
@@ -179,7 +171,10 @@ layernorm_warp_bf16(const __nv_bfloat16 *__restrict__ in, const int32_t *__restr
 // All rows of a bf16 input (no gather), for D <= 8192: one warp per row as in
 // layernorm_warp_bf16, but each warp streams its rows through two shared-memory
 // buffers filled by 1-D bulk copies, the next row's copy in flight while the
-// current row is normalised and written.  Same arithmetic, same bits.
+// current row is normalised and written.  Same arithmetic, same bits.  With
+// scatter_map, row j is also written to out2[scatter_map[j]] when that is
+// >= 0: the LN of every latent (for K and V) then also yields the gathered LN
+// of the active ones (for Q') without reading them a second time.
 constexpr int kBulkWarps = 4;
 
 template <int CPL>
@@ -301,25 +296,23 @@ void launch_bulk_bf16(const __nv_bfloat16 *in, int n_rows, int D, __nv_bfloat16 
 
 template <int CPL>
 void launch_warp_bf16(const __nv_bfloat16 *in, const int32_t *rows, int n_rows, int D,
-                      __nv_bfloat16 *out, const int32_t *scatter_map, __nv_bfloat16 *out2,
-                      cudaStream_t st) {
+                      __nv_bfloat16 *out, cudaStream_t st) {
     constexpr int RPB = kThreads / 32;
     int grid = (n_rows + RPB - 1) / RPB;
     if (grid > 152 * 8) grid = 152 * 8;
-    layernorm_warp_bf16<CPL><<<grid, kThreads, 0, st>>>(in, rows, n_rows, D, out, scatter_map,
-                                                        out2);
+    layernorm_warp_bf16<CPL><<<grid, kThreads, 0, st>>>(in, rows, n_rows, D, out);
 }
 
-void launch_bf16(const __nv_bfloat16 *in, const int32_t *rows, int n_rows, int D,
-                 __nv_bfloat16 *out, const int32_t *scatter_map, __nv_bfloat16 *out2,
-                 cudaStream_t st) {
+// gathered rows of a bf16 input: the row packed in registers
+void launch_gather_bf16(const __nv_bfloat16 *in, const int32_t *rows, int n_rows, int D,
+                        __nv_bfloat16 *out, cudaStream_t st) {
     const int cpl = (D / 8 + 31) / 32;   // 16-byte chunks per lane
-    if (cpl <= 4) return launch_warp_bf16<4>(in, rows, n_rows, D, out, scatter_map, out2, st);
-    if (cpl <= 8) return launch_warp_bf16<8>(in, rows, n_rows, D, out, scatter_map, out2, st);
-    if (cpl <= 16) return launch_warp_bf16<16>(in, rows, n_rows, D, out, scatter_map, out2, st);
-    if (cpl <= 20) return launch_warp_bf16<20>(in, rows, n_rows, D, out, scatter_map, out2, st);
-    if (cpl <= 24) return launch_warp_bf16<24>(in, rows, n_rows, D, out, scatter_map, out2, st);
-    return launch_warp_bf16<32>(in, rows, n_rows, D, out, scatter_map, out2, st);
+    if (cpl <= 4) return launch_warp_bf16<4>(in, rows, n_rows, D, out, st);
+    if (cpl <= 8) return launch_warp_bf16<8>(in, rows, n_rows, D, out, st);
+    if (cpl <= 16) return launch_warp_bf16<16>(in, rows, n_rows, D, out, st);
+    if (cpl <= 20) return launch_warp_bf16<20>(in, rows, n_rows, D, out, st);
+    if (cpl <= 24) return launch_warp_bf16<24>(in, rows, n_rows, D, out, st);
+    return launch_warp_bf16<32>(in, rows, n_rows, D, out, st);
 }
 
 // Every row of an fp32 input: one warp per row, rows streamed through two
@@ -438,7 +431,7 @@ void launch_t(const T *in, const int32_t *rows, int n_rows, int D, __nv_bfloat16
     echo::LaunchScope ls(ECHO_K_LAYERNORM, n_rows, D, (int64_t)sizeof(T), st);
     if constexpr (sizeof(T) == 2) {
         if (!rows) return launch_all_bf16(in, n_rows, D, out, nullptr, nullptr, st);
-        return launch_bf16(in, rows, n_rows, D, out, nullptr, nullptr, st);
+        return launch_gather_bf16(in, rows, n_rows, D, out, st);
     } else {
         if (!rows) return launch_bulk_f32(in, n_rows, D, out, st);
     }
