@@ -382,6 +382,37 @@ def job_tokens_per_s(tokens_per_replica: int, world: int, ms: float) -> float:
     return world * tokens_per_replica / (ms * 1e-3)
 
 
+def copy_overlap(stack, xh, xs_d, rnum, rden, audio_d, n=3):
+    """How much of a pinned host-to-device copy hides behind the step's kernels
+    on this machine: 1 = fully (the copy engine runs beside the SMs), 0 = not at
+    all.  Three steps alone, three copies alone, then both on two streams."""
+    import torch
+    dev = xs_d[0].device
+    main, side = torch.cuda.current_stream(dev), torch.cuda.Stream(dev)
+    xd = torch.empty_like(xs_d[0])
+
+    def steps():
+        for i in range(n):
+            stack.set_audio(audio_d)
+            stack.step(xs_d[i % 2], rnum, rden)
+
+    def copies():
+        with torch.cuda.stream(side):
+            for _ in range(n):
+                xd.copy_(xh, non_blocking=True)
+
+    def wall(f):
+        torch.cuda.synchronize(dev)
+        t = time.perf_counter()
+        f()
+        torch.cuda.synchronize(dev)
+        return time.perf_counter() - t
+    t_s, t_c = wall(steps), wall(copies)
+    t_b = wall(lambda: (copies(), steps()))
+    return {"steps_s": round(t_s, 4), "copies_s": round(t_c, 4), "both_s": round(t_b, 4),
+            "fraction": round(max(0.0, min(1.0, (t_s + t_c - t_b) / t_c)), 3) if t_c > 0 else None}
+
+
 def make_stack(args, w, blocks, dev):
     """The CachedStack of the requested cache form and selection."""
     from paper_2608_02474_gb300 import echocache as ec
@@ -609,6 +640,8 @@ def main():
                "host_ms_per_step": round(host_enqueue_ms, 3)}
         if rate is not None:   # the budgets this leg ran (the rate state carries on)
             e2e["budgets"] = rate.budgets[-args.steps:]
+        else:
+            e2e["copy_overlap"] = copy_overlap(stack, xh[0], xs_d, rnum, rden, audio_d)
 
     cache_bytes = stack.cache_bytes()
     cache_bytes_rs = stack.cache_bytes(right_sized=True)
