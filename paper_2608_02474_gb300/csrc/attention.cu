@@ -8,7 +8,7 @@
 //   warp 0      TMA producer: both Q tiles once, then 128-key blocks K_0, V_0,
 //               K_1, V_1, ... (128-byte swizzle, 64-column boxes) into a ring
 //               shared by K and V (5 slots for d = 128);
-//   warp 1      one thread issues S_t = Q_t K_j^T (M 128, N 128, K d) into the
+//   warp 1      one elected lane issues S_t = Q_t K_j^T (M 128, N 128, K d) into the
 //               tile's TMEM S columns and O_t += P_t V_j (M 128, N d, K 128; P
 //               read from TMEM, V read MN-major straight from its row-major
 //               tile) into the tile's TMEM O accumulator, in the order
@@ -131,58 +131,113 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             for (int li = issued - RING < 0 ? 0 : issued - RING; li < issued; ++li)
                 mbar_wait(&ring_full[li % RING], (li / RING) & 1, abort_v, nullptr, 100000000ull);
         }
-    } else if (warp == 1 && lane == 0) {
+    } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
         // order: S0_0 S1_0 | PV0_0 S0_1 PV1_0 S1_1 | PV0_1 S0_2 PV1_1 S1_2 | ...
-        // Each ring slot is waited for once, before tile 0 uses it: a wait costs
-        // about as much as an MMA even when the data has landed, and this thread
-        // issues tile 1's use of the same slot later.
+        // The whole warp runs this loop and one elected lane issues the MMAs and
+        // commits: the ring arithmetic and the descriptors then stay warp-uniform
+        // and feed tcgen05.mma directly.  Issued from a single diverged lane, the
+        // same loop ran the tensor cores about a quarter slower.
+        // K_{j+1} and V_{j+1} are waited for together, once, before S0_{j+1}:
+        // every wait and fence sits on the path that feeds the tensor cores.
         // P_t lives in the first 64 columns of S_t; S_t of the next block is
         // issued after P V of this block, and tcgen05.mma from one thread run in
         // order, so the S write cannot overtake the P read.  The commit of S_t
         // (s_full) therefore also tells the softmax that P V_{t, j-1} is done.
-        bool ok = mbar_wait(&q_full, 0, abort_v, p.err);
-        auto issue_s = [&](int t, int j) -> bool {
-            const int li = 2 * j, slot = li % RING;
-            if (t == 0) {   // tile 1 uses the slot after tile 0: this thread saw it land
-                if (!mbar_wait(&ring_full[slot], (li / RING) & 1, abort_v, p.err)) return false;
-                tc_fence_after();
-            }
-            const uint8_t *qt = Qs + t * C::Q_BYTES;
-            const uint8_t *kt = Ring + slot * C::SLOT_BYTES;
+        const bool leader = elect_one_sync();
+        // Shared-memory descriptors as two words: the low word holds the start
+        // address in 16-byte units and the leading byte offset, the high word the
+        // 1024-byte stride of eight 128-byte rows, the descriptor version and the
+        // 128-byte swizzle.  A K step only adds a constant to the low word.
+        constexpr uint32_t DESC_HI = (1024u >> 4) | (1u << 14) | (2u << 29);
+        constexpr uint32_t LO_K = 1u << 16;                            // K-major: LBO unused
+        constexpr uint32_t LO_MN = (uint32_t)(ATOM_BYTES >> 4) << 16;  // MN-major: LBO = one atom
+        const uint32_t q_lo = ((smem_u32(Qs) & 0x3FFFFu) >> 4) | LO_K;
+        const uint32_t ring_lo = (smem_u32(Ring) & 0x3FFFFu) >> 4;
+        auto desc = [](uint32_t lo) -> uint64_t { return ((uint64_t)DESC_HI << 32) | lo; };
+        auto wait_all = [&](uint64_t *bar, uint32_t parity) -> bool {
+            return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_v, p.err));
+        };
+        bool ok = wait_all(&q_full, 0);
+        auto mma_s = [&](int t, int slot) {
+            const uint32_t a_lo = q_lo + (uint32_t)t * (C::Q_BYTES >> 4);
+            const uint32_t b_lo = (ring_lo + (uint32_t)slot * (C::SLOT_BYTES >> 4)) | LO_K;
+            const uint32_t d = tmem + (uint32_t)(t * BN);
 #pragma unroll
             for (int kk = 0; kk < DH / 16; ++kk) {
-                const int a = kk >> 2, off = (kk & 3) * 32;
-                tc_mma_f16(tmem + (uint32_t)(t * BN), smem_desc_sw128(qt + a * ATOM_BYTES + off),
-                           smem_desc_sw128(kt + a * ATOM_BYTES + off), C::IDESC_S, kk > 0);
+                const uint32_t off = (uint32_t)(((kk >> 2) * ATOM_BYTES + (kk & 3) * 32) >> 4);
+                tc_mma_f16(d, desc(a_lo + off), desc(b_lo + off), C::IDESC_S, kk > 0);
             }
-            tc_commit(&s_full[t]);
-            if (t == TILES - 1) tc_commit(&ring_empty[slot]);   // K_j no longer needed
-            return true;
         };
-        auto issue_pv = [&](int t, int j) -> bool {
-            const int li = 2 * j + 1, slot = li % RING;
-            if (!mbar_wait(&p_full[t], j & 1, abort_v, p.err)) return false;
-            if (t == 0 && !mbar_wait(&ring_full[slot], (li / RING) & 1, abort_v, p.err)) return false;
-            tc_fence_after();
-            const uint8_t *vt = Ring + slot * C::SLOT_BYTES;
+        auto mma_pv = [&](int t, int slot, uint32_t acc0) {
+            const uint32_t b_lo = (ring_lo + (uint32_t)slot * (C::SLOT_BYTES >> 4)) | LO_MN;
+            const uint32_t d = tmem + O_COL + (uint32_t)(t * DH);
+            const uint32_t a = tmem + (uint32_t)(t * BN);
+            tc_mma_f16_tmem_a(d, a, desc(b_lo), C::IDESC_PV, acc0);
 #pragma unroll
-            for (int kk = 0; kk < BN / 16; ++kk)
-                tc_mma_f16_tmem_a(tmem + O_COL + (uint32_t)(t * DH), tmem + (uint32_t)(t * BN + 8 * kk),
-                                  smem_desc_sw128_mn(vt + kk * 2048, ATOM_BYTES, 1024), C::IDESC_PV,
-                                  (j > 0 || kk > 0) ? 1u : 0u);
-            if (j == nb - 1) tc_commit(&pv_done[t]);            // O_t is final
-            if (t == TILES - 1) tc_commit(&ring_empty[slot]);   // V_j no longer needed
-            return true;
+            for (int kk = 1; kk < BN / 16; ++kk)
+                tc_mma_f16_tmem_a(d, a + 8 * kk, desc(b_lo + (uint32_t)(kk * 2048 >> 4)), C::IDESC_PV, 1u);
         };
-        for (int t = 0; ok && t < TILES; ++t) ok = issue_s(t, 0);
-        for (int j = 0; ok && j < nb; ++j) {
-            for (int t = 0; ok && t < TILES; ++t) {
-                ok = issue_pv(t, j);
-                if (ok && j + 1 < nb) ok = issue_s(t, j + 1);
-            }
+        // ring position (slot, phase parity) of K_j; V_j is the next position
+        int ks = 0;
+        uint32_t kph = 0;
+        auto next = [&](int &slot, uint32_t &ph) { if (++slot == RING) { slot = 0; ph ^= 1u; } };
+        {   // K_0 and V_0, then S_0 of both tiles
+            int vs = ks; uint32_t vph = kph; next(vs, vph);
+            ok = ok && wait_all(&ring_full[ks], kph) && wait_all(&ring_full[vs], vph);
         }
-        if (!ok) {  // wait for the MMAs already issued before tensor memory is freed
+        if (ok) {
+            tc_fence_after();
+            if (leader) {
+                mma_s(0, ks);
+                tc_commit(&s_full[0]);
+                mma_s(1, ks);
+                tc_commit(&s_full[1]);
+                tc_commit(&ring_empty[ks]);
+            }
+            __syncwarp();
+        }
+        for (int j = 0; ok && j < nb; ++j) {
+            int vs = ks; uint32_t vph = kph; next(vs, vph);       // V_j
+            int ns = vs; uint32_t nph = vph; next(ns, nph);       // K_{j+1}
+            int ws = ns; uint32_t wph = nph; next(ws, wph);       // V_{j+1}
+            const bool more = j + 1 < nb;
+            const uint32_t acc0 = j > 0 ? 1u : 0u;
+            // tile 0: P V_j, then S_{j+1} once K_{j+1} and V_{j+1} have landed
+            if (!wait_all(&p_full[0], j & 1)) { ok = false; break; }
+            tc_fence_after();
+            if (leader) {
+                mma_pv(0, vs, acc0);
+                if (!more) tc_commit(&pv_done[0]);
+            }
+            __syncwarp();
+            if (more) {
+                if (!wait_all(&ring_full[ns], nph) || !wait_all(&ring_full[ws], wph)) { ok = false; break; }
+                tc_fence_after();
+                if (leader) {
+                    mma_s(0, ns);
+                    tc_commit(&s_full[0]);
+                }
+                __syncwarp();
+            }
+            // tile 1
+            if (!wait_all(&p_full[1], j & 1)) { ok = false; break; }
+            tc_fence_after();
+            if (leader) {
+                mma_pv(1, vs, acc0);
+                if (!more) tc_commit(&pv_done[1]);
+                tc_commit(&ring_empty[vs]);                      // V_j no longer needed
+                if (more) {
+                    mma_s(1, ns);
+                    tc_commit(&s_full[1]);
+                    tc_commit(&ring_empty[ns]);                  // K_{j+1} no longer needed
+                }
+            }
+            __syncwarp();
+            ks = ns;
+            kph = nph;
+        }
+        if (!ok && leader) {  // wait for the MMAs already issued before tensor memory is freed
             tc_commit(&drain);
             mbar_wait(&drain, 0, abort_v, nullptr, 100000000ull);
         }

@@ -6,7 +6,7 @@
 // 8 warps:
 //   warp 0      TMA producer: A [128 x 64] and W [256 x 64] bf16 tiles, 128-byte
 //               swizzle, into a 4-stage shared-memory ring (48 KB per stage);
-//   warp 1      one thread issues tcgen05.mma (M=128, N=256, K=16) into one of two
+//   warp 1      one elected lane issues tcgen05.mma (M=128, N=256, K=16) into one of two
 //               128 x 256 fp32 accumulators in tensor memory, and commits each
 //               stage back to the producer, so the epilogue of one tile overlaps
 //               the main loop of the next;
@@ -126,13 +126,24 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
             for (int k = it - STAGES < 0 ? 0 : it - STAGES; k < it; ++k)
                 mbar_wait(&full_bar[k % STAGES], (k / STAGES) & 1, abort_v, nullptr, 100000000ull);
         }
-    } else if (warp == 1 && lane == 0) {
+    } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
+        // The whole warp runs the loop (stage arithmetic and descriptors stay
+        // warp-uniform) and one elected lane issues the MMAs and commits.
+        // Descriptor words: the low word holds the start address in 16-byte
+        // units (leading byte offset unused for K-major), the high word the
+        // 1024-byte stride of eight 128-byte rows, the version and the 128-byte
+        // swizzle; a K step of 16 adds 32 bytes to the start address.
+        const bool leader = elect_one_sync();
+        constexpr uint32_t DESC_HI = (1024u >> 4) | (1u << 14) | (2u << 29);
+        const uint32_t smem_lo = ((smem_u32(smem) & 0x3FFFFu) >> 4) | (1u << 16);
+        auto desc = [](uint32_t lo) -> uint64_t { return ((uint64_t)DESC_HI << 32) | lo; };
         bool ok = true;
         int it = 0, local = 0;
         for (int t = blockIdx.x; ok && t < num_tiles; t += gridDim.x, ++local) {
             const int buf = local & 1;
-            if (!mbar_wait(&acc_empty[buf], ((local >> 1) & 1) ^ 1, abort_v, p.err)) {
+            if (!__all_sync(0xffffffffu,
+                            mbar_wait(&acc_empty[buf], ((local >> 1) & 1) ^ 1, abort_v, p.err))) {
                 ok = false;
                 break;
             }
@@ -140,22 +151,25 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
             const uint32_t d_tmem = tmem + (uint32_t)(buf * BN);
             for (int kb = 0; kb < num_kb; ++kb, ++it) {
                 const int s = it % STAGES;
-                if (!mbar_wait(&full_bar[s], (it / STAGES) & 1, abort_v, p.err)) {
+                if (!__all_sync(0xffffffffu, mbar_wait(&full_bar[s], (it / STAGES) & 1, abort_v, p.err))) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint8_t *a = smem + s * STAGE_BYTES;
-                const uint8_t *b = a + A_BYTES;
+                const uint32_t a_lo = smem_lo + (uint32_t)(s * (STAGE_BYTES >> 4));
+                const uint32_t b_lo = a_lo + (uint32_t)(A_BYTES >> 4);
+                if (leader) {
 #pragma unroll
-                for (int k = 0; k < BK / 16; ++k)
-                    tc_mma_f16(d_tmem, smem_desc_sw128(a + k * 32), smem_desc_sw128(b + k * 32), IDESC,
-                               (kb | k) != 0);
-                tc_commit(&empty_bar[s]);
+                    for (int k = 0; k < BK / 16; ++k)
+                        tc_mma_f16(d_tmem, desc(a_lo + 2 * k), desc(b_lo + 2 * k), IDESC, (kb | k) != 0);
+                    tc_commit(&empty_bar[s]);
+                }
+                __syncwarp();
             }
-            if (ok) tc_commit(&acc_full[buf]);
+            if (ok && leader) tc_commit(&acc_full[buf]);
+            __syncwarp();
         }
-        if (!ok) {  // wait for the MMAs already issued before tensor memory is freed
+        if (!ok && leader) {  // wait for the MMAs already issued before tensor memory is freed
             tc_commit(&drain_bar);
             mbar_wait(&drain_bar, 0, abort_v, nullptr, 100000000ull);
         }
