@@ -262,6 +262,10 @@ GEMM_CASES = [
     (1000, 1024, 1024),
     (513, 512, 128),
     (200, 5120, 512),
+    # more 256 x 256 tiles than CTA pairs on the GPU: pairs take several tiles,
+    # alternating their two accumulators, and the 6-stage ring wraps across tiles
+    (2000, 64, 2560),
+    (4100, 320, 1536),
 ]
 
 
