@@ -138,8 +138,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         // commits: the ring arithmetic and the descriptors then stay warp-uniform
         // and feed tcgen05.mma directly.  Issued from a single diverged lane, the
         // same loop ran the tensor cores about a quarter slower.
-        // K_{j+1} and V_{j+1} are waited for together, once, before S0_{j+1}:
-        // every wait and fence sits on the path that feeds the tensor cores.
+        // Every wait and fence sits on the path that feeds the tensor cores:
+        // K_{j+1} is waited for before S0_{j+1}, V_{j+1} after S1_{j+1}.
         // P_t lives in the first 64 columns of S_t; S_t of the next block is
         // issued after P V of this block, and tcgen05.mma from one thread run in
         // order, so the S write cannot overtake the P read.  The commit of S_t
@@ -203,7 +203,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             int ws = ns; uint32_t wph = nph; next(ws, wph);       // V_{j+1}
             const bool more = j + 1 < nb;
             const uint32_t acc0 = j > 0 ? 1u : 0u;
-            // tile 0: P V_j, then S_{j+1} once K_{j+1} and V_{j+1} have landed
+            // tile 0: P V_j, then S_{j+1} once K_{j+1} has landed
             if (!wait_all(&p_full[0], j & 1)) { ok = false; break; }
             tc_fence_after();
             if (leader) {
@@ -212,7 +212,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             }
             __syncwarp();
             if (more) {
-                if (!wait_all(&ring_full[ns], nph) || !wait_all(&ring_full[ws], wph)) { ok = false; break; }
+                if (!wait_all(&ring_full[ns], nph)) { ok = false; break; }
                 tc_fence_after();
                 if (leader) {
                     mma_s(0, ns);
@@ -234,6 +234,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 }
             }
             __syncwarp();
+            // V_{j+1} is read by the next block's P V only.  Waiting for it here
+            // rather than beside K_{j+1} puts the wait in the window in which
+            // tile 0's softmax forms P_{j+1}, and lets S0_{j+1} start sooner.
+            if (more && !wait_all(&ring_full[ws], wph)) { ok = false; break; }
             ks = ns;
             kph = nph;
         }
