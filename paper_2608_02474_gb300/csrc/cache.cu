@@ -116,18 +116,30 @@ quant_amax_kernel(const __nv_bfloat16 *__restrict__ src, const uint32_t *__restr
             sc = __fdiv_rn(amax, 127.f);
             inv = __fdiv_rn(127.f, amax);
         }
-        for (int c = lane; c < C; c += 32) {
-            float f[8];
-            load8<__nv_bfloat16>(s + 8 * c, f);
-            uint32_t w[2] = {0u, 0u};
+        // four 16-byte loads in flight per lane before any of them is used
+        for (int c0 = lane; c0 < C; c0 += 4 * 32) {
+            uint4 u[4];
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                float t = rintf(__fmul_rn(f[k], inv));
-                t = fminf(fmaxf(t, -127.f), 127.f);
-                const uint32_t b = (uint32_t)(uint8_t)(int8_t)(int)t;
-                w[k >> 2] |= b << (8 * (k & 3));
+            for (int i = 0; i < 4; ++i) {
+                const int c = c0 + 32 * i;
+                u[i] = c < C ? __ldcs(reinterpret_cast<const uint4 *>(s + 8 * c)) : make_uint4(0, 0, 0, 0);
             }
-            *reinterpret_cast<uint2 *>(qr + 8 * c) = make_uint2(w[0], w[1]);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int c = c0 + 32 * i;
+                if (c >= C) break;
+                float f[8];
+                unpack8_bf16(u[i], f);
+                uint32_t w[2] = {0u, 0u};
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    float t = rintf(__fmul_rn(f[k], inv));
+                    t = fminf(fmaxf(t, -127.f), 127.f);
+                    const uint32_t b = (uint32_t)(uint8_t)(int8_t)(int)t;
+                    w[k >> 2] |= b << (8 * (k & 3));
+                }
+                *reinterpret_cast<uint2 *>(qr + 8 * c) = make_uint2(w[0], w[1]);
+            }
         }
         if (lane == 0) scale[r] = sc;
     }
