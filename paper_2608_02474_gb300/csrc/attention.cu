@@ -348,22 +348,40 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[t], 0, abort_v, p.err));
         if (ok) {
             tc_fence_after();
-            const int row = q0 + t * BM + r;
             const float inv = 1.f / l;
-            __nv_bfloat16 *dst = p.O + (int64_t)row * p.ldo + h * DH;
+            // The warp's 32 rows of O go through its quarter of Q_t (free now:
+            // every MMA that read Q_t is done) and leave in whole row segments,
+            // CH lanes per row, instead of one row per lane.  The 16-byte chunks
+            // of a staged row are XOR-swizzled by the row so that both the
+            // row-per-lane writes and the chunk-per-lane reads spread over the
+            // shared-memory banks.
+            constexpr int RB = DH * 2, CH = RB / 16;          // bytes and 16-byte chunks per row
+            uint8_t *stage = Qs + t * C::Q_BYTES + quad * 32 * RB;
 #pragma unroll
             for (int c = 0; c < DH / 32; ++c) {
                 uint32_t o[32];
                 tmem_ld32(tmem + lane_base + o_col + 32 * c, o);
                 tmem_ld_wait();
-                if (row < p.M) {
-                    float f[32];
+                float f[32];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) f[i] = __uint_as_float(o[i]) * inv;
-                    uint4 *op = reinterpret_cast<uint4 *>(dst + 32 * c);
+                for (int i = 0; i < 32; ++i) f[i] = __uint_as_float(o[i]) * inv;
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) op[i] = pack8_bf16(f + 8 * i);
+                for (int i = 0; i < 4; ++i) {
+                    const int cc = 4 * c + i;
+                    *reinterpret_cast<uint4 *>(stage + lane * RB + ((cc ^ (lane & (CH - 1))) * 16)) =
+                        pack8_bf16(f + 8 * i);
                 }
+            }
+            __syncwarp();
+            constexpr int RPI = 32 / CH;                        // rows per warp-wide store
+#pragma unroll
+            for (int k = 0; k < 32 / RPI; ++k) {
+                const int rr = k * RPI + lane / CH, cc = lane % CH;
+                const uint4 v =
+                    *reinterpret_cast<const uint4 *>(stage + rr * RB + ((cc ^ (rr & (CH - 1))) * 16));
+                const int grow = q0 + t * BM + quad * 32 + rr;
+                if (grow < p.M)
+                    *reinterpret_cast<uint4 *>(p.O + (int64_t)grow * p.ldo + h * DH + 8 * cc) = v;
             }
         }
     }
