@@ -21,7 +21,7 @@ import torch
 from . import echocache as ec
 
 
-def main():
+def make_parser() -> argparse.ArgumentParser:
     ap = argparse.ArgumentParser()
     ap.add_argument("--kernel", required=True,
                     choices=["gemm", "attention", "drift", "select", "merge", "quant", "layernorm",
@@ -40,7 +40,11 @@ def main():
     ap.add_argument("--samples", type=int, default=80960, help="energy: audio samples")
     ap.add_argument("--iters", type=int, default=3)
     ap.add_argument("--warmup", type=int, default=1)
-    a = ap.parse_args()
+    return ap
+
+
+def main():
+    a = make_parser().parse_args()
 
     dev = torch.device("cuda")
     g = torch.Generator(device=dev).manual_seed(0)
