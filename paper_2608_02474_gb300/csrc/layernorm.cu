@@ -396,7 +396,64 @@ layernorm_bulk_f32(const float *__restrict__ in, int n_rows, int D, __nv_bfloat1
     }
 }
 
+// fp32 rows of up to 8192 values: one CTA of 128 threads per row, the row in
+// registers (thread t holds 16-byte chunks t, t + 128, ...), every load in
+// flight before the first sum.  Sums: each thread's chunks in order, a xor
+// butterfly per warp, then the four warp partials in order.
+constexpr int kRowThreads = 128, kRowChunks = 16;
+
+__global__ void __launch_bounds__(kRowThreads)
+layernorm_row_f32(const float *__restrict__ in, int D, __nv_bfloat16 *__restrict__ out) {
+    __shared__ float red[2][kRowThreads / 32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int C4 = D >> 2;
+    const float4 *row = reinterpret_cast<const float4 *>(in + (int64_t)blockIdx.x * D);
+    float4 v[kRowChunks];
+#pragma unroll
+    for (int k = 0; k < kRowChunks; ++k) {
+        const int c = threadIdx.x + k * kRowThreads;
+        v[k] = c < C4 ? __ldcs(row + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    float s = 0.f;
+#pragma unroll
+    for (int k = 0; k < kRowChunks; ++k) {
+        s += v[k].x; s += v[k].y; s += v[k].z; s += v[k].w;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (lane == 0) red[0][warp] = s;
+    __syncthreads();
+    const float invD = 1.f / (float)D;
+    const float mean = (((red[0][0] + red[0][1]) + red[0][2]) + red[0][3]) * invD;
+    float ss = 0.f;
+#pragma unroll
+    for (int k = 0; k < kRowChunks; ++k) {
+        if (threadIdx.x + k * kRowThreads < C4) {
+            const float a = v[k].x - mean, b = v[k].y - mean, c = v[k].z - mean, d = v[k].w - mean;
+            ss += a * a; ss += b * b; ss += c * c; ss += d * d;
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    if (lane == 0) red[1][warp] = ss;
+    __syncthreads();
+    const float rstd = rsqrtf((((red[1][0] + red[1][1]) + red[1][2]) + red[1][3]) * invD + 1e-6f);
+    uint2 *dst = reinterpret_cast<uint2 *>(out + (int64_t)blockIdx.x * D);
+#pragma unroll
+    for (int k = 0; k < kRowChunks; ++k) {
+        const int c = threadIdx.x + k * kRowThreads;
+        if (c < C4)
+            dst[c] = make_uint2(pack_bf16((v[k].x - mean) * rstd, (v[k].y - mean) * rstd),
+                                pack_bf16((v[k].z - mean) * rstd, (v[k].w - mean) * rstd));
+    }
+}
+
 void launch_bulk_f32(const float *in, int n_rows, int D, __nv_bfloat16 *out, cudaStream_t st) {
+    if (n_rows <= 0) return;
+    if (D <= 4 * kRowThreads * kRowChunks) {   // D <= 8192 (D is a multiple of 8)
+        layernorm_row_f32<<<n_rows, kRowThreads, 0, st>>>(in, D, out);
+        return;
+    }
     const size_t smem = (size_t)kBulkWarpsF32 * 2 * D * sizeof(float);
     static int attr_done[64] = {};
     int dev = 0;
