@@ -315,7 +315,8 @@ void launch_gather_bf16(const __nv_bfloat16 *in, const int32_t *rows, int n_rows
     return launch_warp_bf16<32>(in, rows, n_rows, D, out, st);
 }
 
-// Every row of an fp32 input: one warp per row, rows streamed through two
+// Every row of an fp32 input wider than 8192 values (narrower rows take
+// layernorm_row_f32 below): one warp per row, rows streamed through two
 // shared-memory buffers per warp by 1-D bulk copies (the next row's copy in
 // flight while the current one is normalised), the statistics read from
 // shared memory: per lane, 8-element chunks lane, lane + 32, ... summed in
