@@ -315,88 +315,6 @@ void launch_gather_bf16(const __nv_bfloat16 *in, const int32_t *rows, int n_rows
     return launch_warp_bf16<32>(in, rows, n_rows, D, out, st);
 }
 
-// Every row of an fp32 input wider than 8192 values (narrower rows take
-// layernorm_row_f32 below): one warp per row, rows streamed through two
-// shared-memory buffers per warp by 1-D bulk copies (the next row's copy in
-// flight while the current one is normalised), the statistics read from
-// shared memory: per lane, 8-element chunks lane, lane + 32, ... summed in
-// order, then an xor butterfly.
-constexpr int kBulkWarpsF32 = 2;
-
-__global__ void __launch_bounds__(kBulkWarpsF32 * 32)
-layernorm_bulk_f32(const float *__restrict__ in, int n_rows, int D, __nv_bfloat16 *__restrict__ out,
-                   int *err) {
-    extern __shared__ __align__(128) uint8_t smem_rows[];
-    __shared__ __align__(8) uint64_t bar[kBulkWarpsF32][2];
-    __shared__ int abort_flag;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const uint32_t row_bytes = (uint32_t)D * 4u;
-    uint8_t *buf = smem_rows + (size_t)warp * 2 * row_bytes;
-    if (lane == 0) {
-        mbar_init(&bar[warp][0], 1);
-        mbar_init(&bar[warp][1], 1);
-    }
-    if (threadIdx.x == 0) abort_flag = 0;
-    fence_barrier_init();
-    __syncthreads();
-    volatile int *abort_v = &abort_flag;
-    const int C = D >> 3;
-    const float invD = 1.f / (float)D;
-    const int nw = gridDim.x * kBulkWarpsF32;
-    int j = blockIdx.x * kBulkWarpsF32 + warp;
-    if (j < n_rows && lane == 0) {
-        mbar_arrive_expect_tx(&bar[warp][0], row_bytes);
-        bulk_load_1d(buf, in + (int64_t)j * D, row_bytes, &bar[warp][0]);
-    }
-    for (int it = 0; j < n_rows; ++it, j += nw) {
-        const int b = it & 1;
-        const int jn = j + nw;
-        __syncwarp();   // every lane is done with buffer b ^ 1 (read in the last iteration)
-        if (jn < n_rows && lane == 0) {
-            fence_proxy_async_smem();
-            mbar_arrive_expect_tx(&bar[warp][b ^ 1], row_bytes);
-            bulk_load_1d(buf + (b ^ 1) * row_bytes, in + (int64_t)jn * D, row_bytes,
-                         &bar[warp][b ^ 1]);
-        }
-        if (!__all_sync(0xffffffffu, mbar_wait(&bar[warp][b], (it >> 1) & 1, abort_v, err))) {
-            if (jn < n_rows)   // let the next copy land before the CTA gives up
-                mbar_wait(&bar[warp][b ^ 1], ((it + 1) >> 1) & 1, abort_v, nullptr, 100000000ull);
-            break;
-        }
-        const float4 *row = reinterpret_cast<const float4 *>(buf + b * row_bytes);
-        float s = 0.f;
-        for (int c = lane; c < C; c += 32) {
-            const float4 a = row[2 * c], d = row[2 * c + 1];
-            s += a.x; s += a.y; s += a.z; s += a.w;
-            s += d.x; s += d.y; s += d.z; s += d.w;
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-        const float mean = s * invD;
-        float ss = 0.f;
-        for (int c = lane; c < C; c += 32) {
-            const float4 a = row[2 * c], d = row[2 * c + 1];
-            const float f[8] = {a.x, a.y, a.z, a.w, d.x, d.y, d.z, d.w};
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                const float dlt = f[e] - mean;
-                ss += dlt * dlt;
-            }
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-        const float rstd = rsqrtf(ss * invD + 1e-6f);
-        uint4 *dst = reinterpret_cast<uint4 *>(out + (int64_t)j * D);
-        for (int c = lane; c < C; c += 32) {
-            const float4 a = row[2 * c], d = row[2 * c + 1];
-            float f[8] = {a.x, a.y, a.z, a.w, d.x, d.y, d.z, d.w};
-#pragma unroll
-            for (int e = 0; e < 8; ++e) f[e] = (f[e] - mean) * rstd;
-            dst[c] = pack8_bf16(f);
-        }
-    }
-}
-
 // fp32 rows of up to 8192 values: one CTA of 128 threads per row, the row in
 // registers (thread t holds 16-byte chunks t, t + 128, ...), every load in
 // flight before the first sum.  Sums: each thread's chunks in order, a xor
@@ -449,26 +367,11 @@ layernorm_row_f32(const float *__restrict__ in, int D, __nv_bfloat16 *__restrict
     }
 }
 
-void launch_bulk_f32(const float *in, int n_rows, int D, __nv_bfloat16 *out, cudaStream_t st) {
+// every row of an fp32 input (D <= 8192: echo_layernorm and the block step
+// reject wider rows)
+void launch_all_f32(const float *in, int n_rows, int D, __nv_bfloat16 *out, cudaStream_t st) {
     if (n_rows <= 0) return;
-    if (D <= 4 * kRowThreads * kRowChunks) {   // D <= 8192 (D is a multiple of 8)
-        layernorm_row_f32<<<n_rows, kRowThreads, 0, st>>>(in, D, out);
-        return;
-    }
-    const size_t smem = (size_t)kBulkWarpsF32 * 2 * D * sizeof(float);
-    static int attr_done[64] = {};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-        cudaFuncSetAttribute(layernorm_bulk_f32, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)(kBulkWarpsF32 * 2 * 8192 * sizeof(float)));
-        attr_done[dev] = 1;
-    }
-    const int per_sm = smem <= 72 * 1024 ? 3 : (smem <= 110 * 1024 ? 2 : 1);
-    int grid = (n_rows + kBulkWarpsF32 - 1) / kBulkWarpsF32;
-    if (grid > 152 * per_sm) grid = 152 * per_sm;
-    layernorm_bulk_f32<<<grid, kBulkWarpsF32 * 32, smem, st>>>(in, n_rows, D, out,
-                                                               echo::device_error_ptr());
+    layernorm_row_f32<<<n_rows, kRowThreads, 0, st>>>(in, D, out);
 }
 
 // every row of a bf16 input, optionally also scattered through a map: the
@@ -491,7 +394,7 @@ void launch_t(const T *in, const int32_t *rows, int n_rows, int D, __nv_bfloat16
         if (!rows) return launch_all_bf16(in, n_rows, D, out, nullptr, nullptr, st);
         return launch_gather_bf16(in, rows, n_rows, D, out, st);
     } else {
-        if (!rows) return launch_bulk_f32(in, n_rows, D, out, st);
+        if (!rows) return launch_all_f32(in, n_rows, D, out, st);
     }
     if (C <= 32 * kMaxChunks / 2) {   // D <= 1024: a warp per row
         constexpr int RPB = kThreads / 32;

@@ -41,11 +41,13 @@ def test_roofline_takes_the_largest_measurable_kernel():
             ("gemm_tcgen05", 32760, 10240, 5120, 1.7), ("gemm_tcgen05", 32760, 10240, 5120, 1.7),
             ("segment_energy_fft", 21, 21, 512, 9.0),      # longest, but latency-bound
             ("drift_score", 32760, 5120, 0, 0.08)]
-    out, table = bench.roofline(recs, K, PEAKS)
+    out, table = bench.roofline(recs, K, PEAKS, timed_s=0.13)
     assert out["kernel"] == "attention" and out["bound"] == "tensor"
     flops = 4.0 * 6552 * 32760 * 5120
     assert out["achieved"] == pytest.approx(flops / 2.5e-3 / 1e12, rel=1e-4)
-    assert out["frac"] == pytest.approx(out["achieved"] / PEAKS["bf16_tflops_sustained"], rel=1e-3)
+    # a 0.13 s timed region is held to the burst peak
+    assert out["peak"] == PEAKS["bf16_tflops"] and "burst" in out["peak_source"]
+    assert out["frac"] == pytest.approx(out["achieved"] / PEAKS["bf16_tflops"], rel=1e-3)
     assert out["launch_ms"] == pytest.approx(2.5)
     assert sum(r["share"] for r in table.values()) == pytest.approx(1.0, abs=1e-3)
     assert table["attention[6552x32760x5120]"]["launches"] == 2
@@ -110,3 +112,46 @@ def test_peaks_come_from_the_measured_file():
     d = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
     assert p["source"] == "measured"
     assert p["hbm_gbs"] == d["hbm_gbs"] and p["bf16_tflops_sustained"] == d["bf16_tflops_sustained"]
+
+
+def test_tensor_peak_follows_the_length_of_the_timed_region():
+    assert bench.tensor_peak(PEAKS, 0.13)[0] == PEAKS["bf16_tflops"]
+    assert bench.tensor_peak(PEAKS, None)[0] == PEAKS["bf16_tflops"]
+    assert bench.tensor_peak(PEAKS, bench.SUSTAINED_MIN_S)[0] == PEAKS["bf16_tflops_sustained"]
+    out, _ = bench.roofline([("attention", 6552, 32760, 5120, 2.5)], 6552, PEAKS, timed_s=3.0)
+    assert out["peak"] == PEAKS["bf16_tflops_sustained"] and "sustained" in out["peak_source"]
+
+
+def test_both_arms_print_the_same_config():
+    import argparse
+    from synth import ALL
+    args = argparse.Namespace(adaptive=None, profile="speech", cache="int8", select="energy",
+                              latents="iid", graph=False)
+    w = ALL["wan_block_32760"]
+    c = bench.workload_config(args, w, 1, 5, w.K, 1)
+    assert c == bench.workload_config(args, w, 1, 5, w.K, 1)
+    assert c["workload"] == "wan_block_32760" and c["active_tokens"] == 6552
+    assert c["ratio"] == "1/5" and c["parallelism"] == "replicas1"
+
+
+def test_reference_arm_times_complete_steps_within_its_budget(capsys):
+    """The reference arm on the 256-token workload: every requested step is a
+    complete oracle step, the line reports the steps it timed, the sampled
+    estimate is marked extrapolated and the config equals the GPU arm's."""
+    import argparse
+    from synth import ALL
+    args = argparse.Namespace(adaptive=None, profile="speech", cache="int8", select="energy",
+                              latents="iid", graph=False, steps=2, warmup=1, gpus=1, tau=0.9,
+                              seg_len=0, ref_budget_s=600.0, no_full_runs=True)
+    w = ALL["tiny_256"]
+    bench.run_reference(args, w, w.ratio_num, w.ratio_den, 0, 1)
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["steps"] == 2 and len(line["step_ms"]) == 2
+    assert line["ms_per_step"] * line["steps"] <= 1e3 * 600
+    assert line["cpu_baseline"]["extrapolated"] is False
+    assert line["sampled_estimate"]["extrapolated"] is True
+    assert line["config"] == bench.workload_config(args, w, 1, 4, w.K, 1)
+    # a budget shorter than one step still times exactly one complete step
+    args.ref_budget_s, args.steps = 0.0, 5
+    bench.run_reference(args, w, w.ratio_num, w.ratio_den, 0, 1)
+    assert json.loads(capsys.readouterr().out.strip().splitlines()[-1])["steps"] == 1
