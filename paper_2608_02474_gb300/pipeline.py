@@ -124,6 +124,12 @@ class CachedStack:
         self._audio_key = None
         self.band, self.seg = self._band[0], self._seg[0]
         self.last_K = []
+        # Optional inspection hook, called from the host as each layer is
+        # enqueued: layer_hook("pre", l, x, None, 0, None) before layer l's
+        # selection, layer_hook("post", l, x, idx, K, y) after its block step
+        # (x is the layer's input, y its output).  A hook that reads device
+        # tensors synchronises with the stream; None (the default) costs nothing.
+        self.layer_hook = None
 
     def set_audio(self, audio: torch.Tensor, n_fft: int = 512, hop: int = 160, n_bands: int = 8):
         """Segment energy of the audio (Sec. 3.3) for the next step.  The result
@@ -171,7 +177,10 @@ class CachedStack:
         cur = x
         self.last_K = []
         last = len(self.blocks) - 1
+        hook = self.layer_hook
         for l, blk in enumerate(self.blocks):
+            if hook is not None:
+                hook("pre", l, cur, None, 0, None)
             if full:
                 idx, K = self.all_idx, self.NT
             elif self.selection == "uniform":
@@ -200,6 +209,8 @@ class CachedStack:
                 ec.echo_block_step_cache(blk, self.dims, cur, idx, K, self.caches[l], y=dst,
                                          workspace=self.ws)
             self.last_K.append(K)
+            if hook is not None:
+                hook("post", l, cur, idx, K, dst)
             cur = dst
         return cur
 

@@ -130,6 +130,19 @@ def step_input(w: Workload, x0: np.ndarray, t: int) -> np.ndarray:
     return to_bf16_values(acc)
 
 
+def step_inputs(w: Workload, x0: np.ndarray, steps: int):
+    """The layer-0 inputs of steps 0 .. steps-1 in order: the same values as
+    step_input(w, x0, t) for each t, drawn incrementally (one perturbation per
+    step instead of t)."""
+    acc = x0.astype(np.float32).copy()
+    for t in range(steps):
+        if t:
+            e = rng(100 + t).standard_normal(x0.shape, dtype=np.float32)
+            e *= np.float32(0.05)
+            acc += e
+        yield to_bf16_values(acc)
+
+
 # ---- generic kernel-level inputs (for parity checks of single entry points) ----
 
 def random_rows(n_rows: int, D: int, seed: int, scale: float = 1.0) -> np.ndarray:

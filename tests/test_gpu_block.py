@@ -1,24 +1,38 @@
 """GPU parity of the cached layer step (echo_select + echo_block_step) against the oracle.
 
-Every GPU call is fed the oracle's own state (layer input and cache at that
-step and layer), so the two sides see identical inputs; nothing the GPU
-produced is fed to the oracle.  Bars: selection indices bit-exact, inactive
-rows bit-exact (they are the reconstructed cache), inactive cache rows
-untouched, active rows within a per-token normwise max rel of 2e-2 and a
-mean rel of 5e-3,
-and the cache rows written on the GPU are exactly the quantisation of the
-bf16 rows it returned.
+The GPU and the oracle always see identical inputs.  In the oracle-trajectory
+tests every GPU call is fed the oracle's own state (layer input and cache at
+that step and layer).  In the 40-layer test the GPU runs its own trajectory
+through CachedStack, and at sampled (step, layer) pairs the oracle is fed the
+GPU's layer input, cache and segment energy (teacher forcing, so that bf16
+differences never change a later selection).
+
+Bars: selection indices bit-exact, inactive rows bit-exact (they are the
+reconstructed cache), inactive cache rows untouched, the cache rows written on
+the GPU exactly the quantisation of the bf16 rows it returned; active rows
+within a per-token normwise max rel of 2e-2 and a mean rel of 5e-3, and their
+element-wise relative error (|g - o| / max(|o|, 0.1 rms)) at most EL_FACTOR
+times that of the ideal bf16 tensor-core block (bf16_model) on the same rows.
 """
 import numpy as np
 import pytest
 import torch
 
 import oracle
-from synth import STACK4_7800, TINY_256, WAN_BLOCK_32760, generate as G
+from bf16_model import elementwise_rel, normwise_rel
+import bf16_model as M
+from synth import STACK4_7800, TINY_256, WAN_BLOCK_32760, WAN_STACK40_32760, WAN_SWEEP_63960
+from synth import generate as G
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda"
 F32 = np.float32
+# The GPU's element-wise error may exceed the ideal bf16 block's by this factor:
+# beyond the model's roundings it accumulates in fp32 in tile order, takes exp2
+# from the hardware's approximation, and rounds P to bf16 against a running
+# maximum taken from the first key block rather than the row's true maximum.
+# Measured on GB300 the ratio stayed within 0.86-1.36 over every case here.
+EL_FACTOR = 1.5
 
 
 @pytest.fixture(scope="module")
@@ -32,13 +46,6 @@ def ec():
 
 def bf(a):
     return torch.from_numpy(np.ascontiguousarray(a, dtype=F32)).to(DEV, torch.bfloat16)
-
-
-def rel_err(g, o):
-    """(max over tokens of max_j|g-o| / max_j|o|, sum|g-o| / sum|o|); the
-    normwise reading of "max relative" is justified in test_tolerance_reading.py."""
-    nw = np.abs(g - o).max(axis=-1) / np.abs(o).max(axis=-1)
-    return float(nw.max()), float(np.abs(g - o).sum() / np.abs(o).sum())
 
 
 def gpu_layer(ec, blk, w, x, q, s, e, ratio, full=False):
@@ -56,28 +63,51 @@ def gpu_layer(ec, blk, w, x, q, s, e, ratio, full=False):
     return idx.cpu().numpy(), y, qd, sd
 
 
-def check_layer(ec, w, res, q_in, s_in, g_idx, y, qd, sd, rows=None):
+def check_active(g, o, emu, tag):
+    """Normwise and mean bars, and the element-wise figure against the model's."""
+    mx, mean = normwise_rel(g, o)
+    el = elementwise_rel(g, o)
+    el_m = elementwise_rel(emu, o)
+    print(f"[{tag}] rows {len(o)}: normwise {mx:.3e}  mean {mean:.3e}  elementwise {el:.3e}  "
+          f"(ideal bf16 {el_m:.3e}, ratio {el / el_m:.2f})")
+    assert mx <= 2e-2 and mean <= 5e-3, (tag, mx, mean)
+    assert el <= EL_FACTOR * el_m, (tag, el, el_m)
+    return mx, mean, el, el_m
+
+
+def check_cache_and_inactive(ec, w, idx, q_in, s_in, g, y, gq, gs):
+    """Inactive rows = the reconstructed cache, bit for bit; inactive cache rows
+    untouched; the written cache rows = echo_cache_quant of the rows returned
+    (echo_cache_quant is itself pinned bit-exact to the oracle)."""
+    inactive = np.setdiff1d(np.arange(w.NT), idx)
+    ref_inactive = oracle.cache.dequantize_rows(q_in[inactive], s_in[inactive])
+    assert np.array_equal(g[inactive], ref_inactive)
+    assert np.array_equal(gq[inactive], q_in[inactive]) and np.array_equal(gs[inactive], s_in[inactive])
+    if len(idx):
+        it = torch.from_numpy(idx.astype(np.int64)).to(DEV)
+        q2 = torch.empty(len(idx), w.D, dtype=torch.int8, device=DEV)
+        s2 = torch.empty(len(idx), dtype=torch.float32, device=DEV)
+        ec.echo_cache_quant(y[it].contiguous(), None, q2, s2)
+        assert np.array_equal(gq[idx], q2.cpu().numpy())
+        assert np.array_equal(gs[idx], s2.cpu().numpy())
+
+
+def check_layer(ec, w, res, q_in, s_in, g_idx, y, qd, sd, emu, tag, rows=None):
     assert np.array_equal(g_idx, res.idx)
     g = y.float().cpu().numpy()
     act = res.idx if rows is None else rows
     ya = res.y_act if rows is None else res.y_act_rows
-    mx, mean = rel_err(g[act], ya)
-    assert mx <= 2e-2 and mean <= 5e-3, (mx, mean)
-    inactive = np.setdiff1d(np.arange(w.NT), res.idx)
-    ref_inactive = oracle.cache.dequantize_rows(q_in[inactive], s_in[inactive])
-    assert np.array_equal(g[inactive], ref_inactive)
-    gq, gs = qd.cpu().numpy(), sd.cpu().numpy()
-    assert np.array_equal(gq[inactive], q_in[inactive]) and np.array_equal(gs[inactive], s_in[inactive])
-    # cache rows written by the step == echo_cache_quant of the bf16 rows it
-    # returned (echo_cache_quant is itself pinned bit-exact to the oracle)
-    if len(res.idx):
-        it = torch.from_numpy(res.idx.astype(np.int64)).to(DEV)
-        q2 = torch.empty(len(res.idx), w.D, dtype=torch.int8, device=DEV)
-        s2 = torch.empty(len(res.idx), dtype=torch.float32, device=DEV)
-        ec.echo_cache_quant(y[it].contiguous(), None, q2, s2)
-        assert np.array_equal(gq[res.idx], q2.cpu().numpy())
-        assert np.array_equal(gs[res.idx], s2.cpu().numpy())
-    return mx, mean
+    out = check_active(g[act], ya, emu, tag)
+    check_cache_and_inactive(ec, w, res.idx, q_in, s_in, g, y, qd.cpu().numpy(), sd.cpu().numpy())
+    return out
+
+
+def _sample_rows(idx, scores, n=32, seed=0):
+    """n rows of idx at random and the n of highest score (scores indexed by
+    the values of idx), ascending and without repeats."""
+    rng = np.random.default_rng(seed)
+    top = idx[np.argsort(-scores[idx], kind="stable")[:n]]
+    return np.unique(np.concatenate([rng.choice(idx, min(n, len(idx)), replace=False), top]))
 
 
 def _trajectory(w, steps, layers, profile="speech"):
@@ -86,42 +116,50 @@ def _trajectory(w, steps, layers, profile="speech"):
     e32 = e.astype(F32)
     Ws = [G.block_weights(w, l) for l in range(layers)]
     cond = G.cond_tokens(w, audio)
-    x0 = G.latents(w)
-    xs = [x0] + [G.step_input(w, x0, t) for t in range(1, steps)]
+    xs = list(G.step_inputs(w, G.latents(w), steps))
     rec = []
     oracle.step.generation(xs, Ws, [cond] * layers, e32, w.T, w.N, w.H, w.ratio_num, w.ratio_den,
                            record=lambda t, l, x, q, s, r: rec.append((t, l, x, q.copy(), s.copy(), r)))
     return Ws, cond, e32, rec
 
 
-def test_tiny_every_step(ec):
-    w = TINY_256
-    Ws, cond, e32, rec = _trajectory(w, w.steps, w.layers)
-    blk = ec.DeviceBlock.from_host(Ws[0], cond)
-    for t, l, x, q, s, r in rec:
-        g_idx, y, qd, sd = gpu_layer(ec, blk, w, x, q, s, e32, (w.ratio_num, w.ratio_den),
-                                     full=t == 0)
-        check_layer(ec, w, r, q, s, g_idx, y, qd, sd)
-
-
-def test_stack4_first_steps(ec):
-    w = STACK4_7800
-    Ws, cond, e32, rec = _trajectory(w, 3, w.layers)
+def _run_trajectory(ec, w, steps, layers, profile="speech", el_rows=256):
+    """Every (step, layer) of the oracle's trajectory; all active rows at the
+    normwise and mean bars, and up to `el_rows` of them (half at random, half
+    of highest score) for the element-wise comparison with the model."""
+    Ws, cond, e32, rec = _trajectory(w, steps, layers, profile)
     blks = [ec.DeviceBlock.from_host(W, cond) for W in Ws]
     for t, l, x, q, s, r in rec:
         g_idx, y, qd, sd = gpu_layer(ec, blks[l], w, x, q, s, e32, (w.ratio_num, w.ratio_den),
                                      full=t == 0)
-        check_layer(ec, w, r, q, s, g_idx, y, qd, sd)
+        tag = f"{w.name} t={t} l={l}"
+        assert np.array_equal(g_idx, r.idx)
+        g = y.float().cpu().numpy()
+        mx, mean = normwise_rel(g[r.idx], r.y_act)
+        assert mx <= 2e-2 and mean <= 5e-3, (tag, mx, mean)
+        j = np.arange(len(r.idx))
+        if len(j) > el_rows:
+            j = _sample_rows(j, r.scores[r.idx] if t else np.zeros(len(j), F32), n=el_rows // 2)
+        emu = M.block_active(x, r.idx[j], Ws[l], cond, w.H)
+        check_active(g[r.idx[j]], r.y_act[j], emu, tag)
+        check_cache_and_inactive(ec, w, r.idx, q, s, g, y, qd.cpu().numpy(), sd.cpu().numpy())
+
+
+def test_tiny_every_step(ec):
+    """The 256-token block over all 8 steps (step 0 full)."""
+    _run_trajectory(ec, TINY_256, TINY_256.steps, TINY_256.layers)
+
+
+def test_stack4_every_step(ec):
+    """The 7800-token, 4-block stack over all 10 steps: from step 2 on the
+    caches hold rows of different ages, and the selection decides which of them
+    are refreshed."""
+    _run_trajectory(ec, STACK4_7800, STACK4_7800.steps, STACK4_7800.layers)
 
 
 @pytest.mark.parametrize("profile", ["silence", "tone", "beats"])
 def test_tiny_profiles(ec, profile):
-    w = TINY_256
-    Ws, cond, e32, rec = _trajectory(w, 3, 1, profile)
-    blk = ec.DeviceBlock.from_host(Ws[0], cond)
-    for t, l, x, q, s, r in rec[1:]:
-        g_idx, y, qd, sd = gpu_layer(ec, blk, w, x, q, s, e32, (w.ratio_num, w.ratio_den))
-        check_layer(ec, w, r, q, s, g_idx, y, qd, sd)
+    _run_trajectory(ec, TINY_256, 3, 1, profile)
 
 
 def test_edge_ratios_and_aliasing(ec):
@@ -140,59 +178,147 @@ def test_edge_ratios_and_aliasing(ec):
     assert np.array_equal(y.float().cpu().numpy(), oracle.cache.dequantize_rows(q, s))
     assert np.array_equal(qd.cpu().numpy(), q)
     # K = NT equals the uncached block; y may alias x
-    r = oracle.step.cached_layer_step(x, q, s, e, W, cond, w.T, w.N, w.H, 1, 1)
     xd = bf(x)
     qd, sd = torch.from_numpy(q.copy()).to(DEV), torch.from_numpy(s.copy()).to(DEV)
     idx = torch.arange(w.NT, dtype=torch.int32, device=DEV)
     ec.echo_block_step(blk, dims, xd, idx, w.NT, qd, sd, y=xd)
-    mx, mean = rel_err(xd.float().cpu().numpy(), oracle.block.uncached_block(x, W, cond, w.H))
-    assert mx <= 2e-2 and mean <= 5e-3
+    check_active(xd.float().cpu().numpy(), oracle.block.uncached_block(x, W, cond, w.H),
+                 M.block_active(x, np.arange(w.NT), W, cond, w.H), "tiny K=NT aliased")
     assert ec.echo_get_device_error() == 0
 
 
+# ---------------------------------------------------------------------------
+# Full-size Wan2.2-S2V-shaped blocks (D 5120, 40 heads x 128, FFN 13824, 672
+# audio tokens).  The oracle recomputes K/V over every token and the block for
+# 64 sampled active rows: 32 at random and the 32 of highest score.
+
+
+
+class _Sampled:
+    """The oracle's sampled rows of one cached layer step."""
+
+    def __init__(self, x, q, s, e32, w, W, cond, ratio, kv=None):
+        self.idx, sc = oracle.select.select(x, q, s, e32, w.T, w.N, *ratio)
+        self.rows = _sample_rows(self.idx, sc)
+        Kv, Vv, Km, Vm = kv if kv is not None else (*oracle.block.self_kv(x, W),
+                                                    *M.self_kv(x, W, fp32=True))
+        Kc, Vc = oracle.block.cross_kv(cond, W)
+        self.y_act_rows = oracle.block.active_rows(x, self.rows, W, w.H, Kv, Vv, Kc, Vc)
+        self.emu = M.active_rows(x, self.rows, W, w.H, Km, Vm, *M.cross_kv(cond, W))
+
+
 @pytest.mark.slow
-@pytest.mark.parametrize("name,layer,step", [("wan_block_32760", 0, 1),
-                                             ("wan_stack40_32760", 39, 1),
-                                             ("wan_stack40_32760", 19, 10),
-                                             ("wan_stack40_32760", 0, 19),
-                                             ("wan_sweep_63960", 0, 1)])
-def test_wan_block_sampled_rows(ec, name, layer, step):
-    """Full-size Wan2.2-S2V-shaped blocks (D 5120, 40 heads) at r = 1/5: the
-    32760-token block, layers 0, 19 and 39 of the 40-layer stack (each with its
-    own weights) at steps 1, 10 and 19, and the 63960-token sweep shape.  Each
-    case is teacher-forced: the layer input is the step-t input and the cache
-    holds the quantised step-(t-1) input, as if that had been the previous
-    output.  Indices bit-exact, inactive rows bit-exact, 64 sampled active rows
-    (32 random, 32 of highest score) against the oracle with keys/values over
-    all tokens."""
-    from synth import ALL
-    w = ALL[name]
+def test_wan_block_sampled_rows(ec):
+    """The 32760-token block at r = 1/5: step-1 input against the quantised
+    step-0 latents, as after the full warm-up step."""
+    w = WAN_BLOCK_32760
     audio = G.audio(w)
-    _, e = oracle.energy.audio_energy(audio, w.T)
-    e32 = e.astype(F32)
-    W = G.block_weights(w, layer)
+    e32 = oracle.energy.audio_energy(audio, w.T)[1].astype(F32)
+    W = G.block_weights(w, 0)
     cond = G.cond_tokens(w, audio)
     x0 = G.latents(w)
-    prev = x0 if step == 1 else G.step_input(w, x0, step - 1)
-    x1 = G.step_input(w, x0, step)
-    q, s, _ = oracle.cache.quantize_rows(prev)    # cache as if the previous output were prev
-    blk = ec.DeviceBlock.from_host(W, cond)
-    g_idx, y, qd, sd = gpu_layer(ec, blk, w, x1, q, s, e32, (w.ratio_num, w.ratio_den))
+    x1 = G.step_input(w, x0, 1)
+    q, s, _ = oracle.cache.quantize_rows(x0)
+    g_idx, y, qd, sd = gpu_layer(ec, ec.DeviceBlock.from_host(W, cond), w, x1, q, s, e32,
+                                 (w.ratio_num, w.ratio_den))
+    o = _Sampled(x1, q, s, e32, w, W, cond, (w.ratio_num, w.ratio_den))
+    check_layer(ec, w, o, q, s, g_idx, y, qd, sd, o.emu, "wan_block_32760", rows=o.rows)
 
-    oidx, osc = oracle.select.select(x1, q, s, e32, w.T, w.N, w.ratio_num, w.ratio_den)
-    assert np.array_equal(g_idx, oidx)
-    rng = np.random.default_rng(0)
-    top = oidx[np.argsort(-osc[oidx], kind="stable")[:32]]
-    rows = np.unique(np.concatenate([rng.choice(oidx, 32, replace=False), top]))
-    Kv, Vv = oracle.block.self_kv(x1, W)
-    Kc, Vc = oracle.block.cross_kv(cond, W)
-    ya = oracle.block.active_rows(x1, rows, W, w.H, Kv, Vv, Kc, Vc)
 
-    class R:
-        pass
-    res = R()
-    res.idx, res.y_act_rows = oidx, ya
-    check_layer(ec, w, res, q, s, g_idx, y, qd, sd, rows=rows)
+@pytest.fixture(scope="module")
+def sweep_state():
+    """63960-token block: the step-1 input, the cache of the quantised step-0
+    latents, and the oracle's and the model's K/V over every token (these
+    depend on neither the ratio nor the audio, so every case shares them)."""
+    w = WAN_SWEEP_63960
+    W = G.block_weights(w, 0)
+    x0 = G.latents(w)
+    x1 = G.step_input(w, x0, 1)
+    q, s, _ = oracle.cache.quantize_rows(x0)
+    del x0
+    kv = (*oracle.block.self_kv(x1, W), *M.self_kv(x1, W, fp32=True))
+    return w, W, x1, q, s, kv
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("profile,ratio", [("speech", (1, 20)), ("speech", (1, 10)),
+                                           ("speech", (1, 5)), ("speech", (1, 2)),
+                                           ("speech", (1, 1)), ("silence", (1, 5)),
+                                           ("tone", (1, 5)), ("beats", (1, 5))],
+                         ids=lambda v: v if isinstance(v, str) else f"r{v[0]}_{v[1]}")
+def test_sweep_63960_sampled_rows(ec, sweep_state, profile, ratio):
+    """The 161-frame sweep block (41 x 30 x 52 = 63960 tokens) at every ratio of
+    the sweep with speech audio, and at r = 1/5 with the silence, tone and
+    beats profiles (which change the segment weights and so the selection).
+    r = 1/20 gives the thinnest attention grid (3198 queries), r = 1 refreshes
+    every token."""
+    w, W, x1, q, s, kv = sweep_state
+    audio = G.audio(w, profile)
+    e32 = oracle.energy.audio_energy(audio, w.T)[1].astype(F32)
+    cond = G.cond_tokens(w, audio)
+    g_idx, y, qd, sd = gpu_layer(ec, ec.DeviceBlock.from_host(W, cond), w, x1, q, s, e32, ratio)
+    o = _Sampled(x1, q, s, e32, w, W, cond, ratio, kv=kv)
+    assert len(o.idx) == oracle.select.refresh_budget(w.NT, *ratio)
+    check_layer(ec, w, o, q, s, g_idx, y, qd, sd, o.emu,
+                f"sweep_63960 {profile} r={ratio[0]}/{ratio[1]}", rows=o.rows)
+
+
+@pytest.mark.slow
+def test_stack40_gpu_trajectory(ec):
+    """The 40-layer stack over 20 steps on the GPU's own trajectory
+    (CachedStack: step 0 full, then r = 1/5 per step and per layer).  At steps
+    {1, 10, 19} x layers {0, 19, 39} the GPU's layer input, its cache before the
+    step and its segment energy are copied to the host and fed to the oracle:
+    indices and inactive rows bit-exact, 64 sampled active rows at the bars.  By
+    step 19 the cache holds rows written at many different steps, each with the
+    scale the FFN-down epilogue's row maximum gave it."""
+    from paper_2608_02474_gb300.pipeline import CachedStack
+    w = WAN_STACK40_32760
+    steps, check_steps, check_layers = w.steps, (1, 10, 19), (0, 19, 39)
+    audio = G.audio(w)
+    cond = G.cond_tokens(w, audio)
+    blocks, Wk = [], {}
+    for l in range(w.layers):
+        W = G.block_weights(w, l)
+        if l in check_layers:
+            Wk[l] = W
+        blocks.append(ec.DeviceBlock.from_host(W, cond))
+        del W
+    st = CachedStack(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc, blocks, device=DEV)
+    st.set_audio(torch.from_numpy(audio).to(DEV))
+    st.wait_audio()
+    e_gpu = st.seg.cpu().numpy().copy()
+    e_ref = oracle.energy.audio_energy(audio, w.T)[1]
+    assert np.all(np.abs(e_gpu - e_ref) <= 1e-5 * np.abs(e_ref))
+    cur = {"t": 0}
+    snap = {}
+    done = []
+
+    def hook(phase, l, x, idx, K, y):
+        if cur["t"] not in check_steps or l not in check_layers:
+            return
+        if phase == "pre":
+            torch.cuda.synchronize()
+            snap["x"] = x.float().cpu().numpy()
+            snap["q"] = st.cache_q[l].cpu().numpy()
+            snap["s"] = st.cache_s[l].cpu().numpy()
+            return
+        torch.cuda.synchronize()
+        assert ec.echo_get_device_error() == 0
+        g_idx = idx[:K].cpu().numpy()
+        o = _Sampled(snap["x"], snap["q"], snap["s"], e_gpu, w, Wk[l], cond,
+                     (w.ratio_num, w.ratio_den))
+        check_layer(ec, w, o, snap["q"], snap["s"], g_idx, y, st.cache_q[l], st.cache_s[l],
+                    o.emu, f"stack40 t={cur['t']} l={l}", rows=o.rows)
+        done.append((cur["t"], l))
+
+    st.layer_hook = hook
+    for t, x in enumerate(G.step_inputs(w, G.latents(w), steps)):
+        cur["t"] = t
+        st.step(bf(x), w.ratio_num, w.ratio_den, full=t == 0)
+    torch.cuda.synchronize()
+    assert ec.echo_get_device_error() == 0
+    assert done == [(t, l) for t in check_steps for l in check_layers]
 
 
 def test_pipeline_host_buffers_match_device_steps(ec):
