@@ -170,8 +170,10 @@ echo_status echo_select(const void *x, echo_dtype xt, const int8_t *cache_q,
  *   workspace; T * N must not exceed ECHO_SELECT_STATIC_MAX_TOKENS, otherwise
  *   ECHO_ERR_WORKSPACE is returned and nothing is enqueued.
  *   The first call on a device looks up that device's address of the array
- *   (once, with the device current); make that first call before any CUDA
- *   stream capture.
+ *   (once, with the device current) and keeps it for the life of the
+ *   process; make that first call before any CUDA stream capture.  A device
+ *   reset (cudaDeviceReset, or anything else that destroys the primary
+ *   context) is not supported: the kept address would then be stale.
  *   All calls on a device share the one array and it keeps the last call's
  *   scores; nothing in it needs to start at zero, because every score the
  *   top-K reads is written first by the same call.  Calls whose work overlaps
@@ -440,7 +442,7 @@ typedef enum {
     ECHO_K_LAYERNORM = 4, ECHO_K_GEMM = 5, ECHO_K_ATTENTION = 6, ECHO_K_QUANT = 7,
     ECHO_K_DEQUANT = 8, ECHO_K_MERGE = 9, ECHO_K_STEP_DELTA = 10, ECHO_K_UNIFORM = 11,
     ECHO_K_REF_SCAN = 12, ECHO_K_REF_ALLOC = 13, ECHO_K_REF_STORE = 14, ECHO_K_CACHE_COPY = 15,
-    ECHO_K_COUNT = 16
+    ECHO_K_MERGE_QUANT = 16, ECHO_K_COUNT = 17
 } echo_kernel_kind;
 
 /* Number of kernels this library has launched in this process (all devices). */
@@ -458,7 +460,8 @@ echo_status echo_profile_enable(int32_t on);
  * H * d); DRIFT (NT, D, 0); TOPK (NT, K, 0); LAYERNORM (rows, D, input element
  * bytes); QUANT, DEQUANT, MERGE (rows, D, 0); ENERGY (T, frames, n_fft); STEP_DELTA (n, element bytes, 0)
  * for the reduction and (0, 0, blocks) for its final combine; UNIFORM (NT, K, 0);
- * REF_SCAN, REF_ALLOC, REF_STORE, CACHE_COPY (rows, D, 0). */
+ * REF_SCAN, REF_ALLOC, REF_STORE, CACHE_COPY (rows, D, 0); MERGE_QUANT (NT, D, K active
+ * rows). */
 int32_t echo_profile_read(int32_t max, int32_t *kinds, int64_t *m, int64_t *n, int64_t *k,
                           float *ms);
 

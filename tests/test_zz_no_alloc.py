@@ -10,6 +10,8 @@ The test calls it through the C ABI twice in a row, on different inputs and
 sizes (the second call reuses the array the first one filled), and checks
 that each call selects exactly the indices echo_select selects with a
 workspace (indices are compared bit-exact, as in every selection test).
+A third case at 63960 tokens reaches the top-K path that keeps its keys in
+global memory and is also compared with the oracle's selection directly.
 This file is collected last so that a failure here never hides another test.
 """
 import ctypes
@@ -65,6 +67,27 @@ def test_static_select_matches_workspace_select_on_two_calls(ec):
         torch.cuda.synchronize()
         assert K == K_ref
         assert np.array_equal(got.cpu().numpy(), ref.cpu().numpy())
+    assert ec.echo_get_device_error() == 0
+
+
+def test_static_select_keys_in_global_memory_match_the_oracle(ec):
+    """41 x 1560 = 63960 tokens (the 161-frame sweep shape, at a small width):
+    more keys than the top-K keeps in shared memory, so the selection keeps them
+    in global memory.  Two calls in a row (r = 1/20, then r = 1/2), each
+    compared bit for bit with echo_select and with the oracle's selection."""
+    import oracle
+    T, N, D = 41, 1560, 64
+    x, q, s, e = _inputs(T, N, D, 21)
+    xh, qh, sh, eh = (t.float().cpu().numpy() if t.dtype == torch.bfloat16 else t.cpu().numpy()
+                      for t in (x, q, s, e))
+    for ratio in ((1, 20), (1, 2)):
+        got, K = _select_static(ec, x, q, s, e, T, N, ratio)
+        ref, K_ref, _ = ec.echo_select(x, q, s, e, T, N, *ratio)
+        torch.cuda.synchronize()
+        o_idx, _ = oracle.select.select(xh, qh, sh, eh, T, N, *ratio)
+        assert K == K_ref == len(o_idx)
+        assert np.array_equal(got.cpu().numpy(), ref.cpu().numpy())
+        assert np.array_equal(got.cpu().numpy(), o_idx)
     assert ec.echo_get_device_error() == 0
 
 
