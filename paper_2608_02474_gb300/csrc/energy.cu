@@ -4,7 +4,10 @@
 // P_k = c_k |X_k|^2 / n_fft is summed over the segment's frames per bin and then
 // per linear band; energy = sqrt(sum of the bands).
 //
-// One CTA per segment, eight frame groups of 128 threads.  Each thread keeps
+// n_fft <= 512 takes the warp kernel below (two frames per complex FFT, the
+// transform in registers and warp shuffles).  Larger transforms take the
+// shared-memory kernel: one CTA per segment, eight frame groups of 128
+// threads.  Each thread keeps
 // the frame-summed power of its bins in registers, so the result does not
 // depend on scheduling: groups are combined in a fixed order and bands are
 // reduced by warps in a fixed order.
@@ -121,6 +124,169 @@ segment_energy_kernel(const float *__restrict__ audio, int seg_len, int n_fft, i
     }
 }
 
+// ---------------------------------------------------------------------------
+// n_fft = 32 R <= 512: one warp transforms two frames at once, no block-wide
+// barrier inside the transform.  The two windowed real frames a and b of a
+// segment are packed as z = a + i b and one complex N-point FFT is taken,
+// N = R x 32 (Cooley-Tukey with N1 = R, N2 = 32): lane n2 holds z[32 n1 + n2]
+// for n1 < R in registers (coalesced loads), takes the R-point DFT over n1 in
+// registers (radix-2, decimation in frequency), multiplies by W_N^(n2 k1), and
+// the 32-point DFT over n2 runs across the lanes (five xor-shuffle radix-2
+// stages).  Lane l then holds Z[k1 + R k2] with k2 = bitrev5(l), k1 = bitrev_R(i)
+// for its register i.  Because a and b are real, |A_k|^2 + |B_k|^2 =
+// (|Z_k|^2 + |Z_{N-k}|^2) / 2, so the summed one-sided power of the two frames
+// at bin k is (|Z_k|^2 + |Z_{N-k}|^2) / N for 0 < k < N/2 and |Z_k|^2 / N at
+// k = 0 and N/2: every Z_k adds |Z_k|^2 / N to bin min(k, N - k), and no value
+// has to meet its mirror image inside the transform.  A lone last frame takes
+// b = 0 (then |Z_{N-k}| = |Z_k|).  Each lane sums |Z|^2 over the pairs its warp
+// takes (pair p goes to warp p mod warps); the warps are combined, the mirror
+// bins folded and the bands reduced in a fixed order.
+// ---------------------------------------------------------------------------
+constexpr int kWarpEnergyWarps = 8;
+
+// W_16^m = exp(-2 pi i m / 16) for m = 0..7: cos(m pi / 8) - i sin(m pi / 8)
+// (cos(pi/8) = sqrt(2 + sqrt 2) / 2, cos(pi/4) = sqrt(2) / 2, cos(3 pi/8) =
+// sqrt(2 - sqrt 2) / 2); folded to immediates in the unrolled loops
+__host__ __device__ constexpr float w16_cos(int m) {
+    return m == 0 ? 1.f : m == 1 ? 0.92387953251128674f : m == 2 ? 0.70710678118654752f
+         : m == 3 ? 0.38268343236508977f : m == 4 ? 0.f : m == 5 ? -0.38268343236508977f
+         : m == 6 ? -0.70710678118654752f : -0.92387953251128674f;
+}
+__host__ __device__ constexpr float w16_sin(int m) { return w16_cos(m >= 4 ? m - 4 : 4 - m); }
+
+ECHO_DEV float2 cmul(float2 a, float2 b) {
+    return make_float2(a.x * b.x - a.y * b.y, a.x * b.y + a.y * b.x);
+}
+
+template <int R>
+__global__ void __launch_bounds__(kWarpEnergyWarps * 32)
+segment_energy_warp_kernel(const float *__restrict__ audio, int seg_len, int hop, int n_frames,
+                           int n_bands, float *__restrict__ band_out, float *__restrict__ seg_out) {
+    constexpr int N = 32 * R, HALF = N / 2;
+    constexpr int LOG2R = R == 2 ? 1 : R == 4 ? 2 : R == 8 ? 3 : 4;
+    static_assert(R == 2 || R == 4 || R == 8 || R == 16, "R-point DFT in registers: R <= 16");
+    __shared__ float win[N];                          // periodic Hann window
+    __shared__ float2 tw2[R][32];                     // W_N^(n2 bitrev_R(i)) for lane n2, register i
+    __shared__ float acc_sh[kWarpEnergyWarps][N];     // per warp, by full-spectrum index
+    __shared__ float bins[HALF + 1];
+    __shared__ float bands[64];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int tau = blockIdx.x;
+    const float *seg = audio + (int64_t)tau * seg_len;
+
+    for (int n = threadIdx.x; n < N; n += blockDim.x) win[n] = 0.5f - 0.5f * cospif((2.0f * n) / N);
+    for (int e = threadIdx.x; e < R * 32; e += blockDim.x) {
+        const int i = e / 32, n2 = e % 32;
+        const int k1 = (int)(__brev((unsigned)i) >> (32 - LOG2R));
+        float sn, cs;
+        sincospif((2.0f * (float)(n2 * k1)) / N, &sn, &cs);
+        tw2[i][n2] = make_float2(cs, -sn);
+    }
+    // cross-lane stage st (half size h = 16 >> st): the upper lane of a pair
+    // multiplies by W_{2h}^(lane mod h); the lower lane by 1
+    float2 twl[5];
+#pragma unroll
+    for (int st = 0; st < 5; ++st) {
+        const int h = 16 >> st;
+        if (lane & h) {
+            float sn, cs;
+            sincospif((float)(lane & (h - 1)) / (float)h, &sn, &cs);
+            twl[st] = make_float2(cs, -sn);
+        } else {
+            twl[st] = make_float2(1.f, 0.f);
+        }
+    }
+    __syncthreads();
+
+    float acc[R];
+#pragma unroll
+    for (int i = 0; i < R; ++i) acc[i] = 0.f;
+    const int n_pairs = (n_frames + 1) >> 1;
+    for (int pr = warp; pr < n_pairs; pr += kWarpEnergyWarps) {
+        const int off_a = 2 * pr * hop, off_b = off_a + hop;
+        const bool has_b = 2 * pr + 1 < n_frames;
+        float2 v[R];
+#pragma unroll
+        for (int n1 = 0; n1 < R; ++n1) {
+            const int n = 32 * n1 + lane;
+            const float w = win[n];
+            const float xa = off_a + n < seg_len ? seg[off_a + n] : 0.f;
+            const float xb = has_b && off_b + n < seg_len ? seg[off_b + n] : 0.f;
+            v[n1] = make_float2(xa * w, xb * w);
+        }
+        // R-point DFT over n1 in registers (output in bit-reversed order)
+#pragma unroll
+        for (int h = R / 2; h >= 1; h >>= 1) {
+#pragma unroll
+            for (int s0 = 0; s0 < R; s0 += 2 * h) {
+#pragma unroll
+                for (int j = 0; j < h; ++j) {
+                    const float2 u = v[s0 + j], x = v[s0 + j + h];
+                    v[s0 + j] = make_float2(u.x + x.x, u.y + x.y);
+                    const int m = j * (16 / (2 * h));          // W_{2h}^j = W_16^(j 16 / 2h)
+                    v[s0 + j + h] = cmul(make_float2(u.x - x.x, u.y - x.y),
+                                         make_float2(w16_cos(m), -w16_sin(m)));
+                }
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < R; ++i) v[i] = cmul(v[i], tw2[i][lane]);
+        // 32-point DFT over n2 across the lanes (output lane = bitrev5(k2))
+#pragma unroll
+        for (int st = 0; st < 5; ++st) {
+            const int h = 16 >> st;
+            const bool upper = (lane & h) != 0;
+#pragma unroll
+            for (int i = 0; i < R; ++i) {
+                const float px = __shfl_xor_sync(0xffffffffu, v[i].x, h);
+                const float py = __shfl_xor_sync(0xffffffffu, v[i].y, h);
+                const float2 d = upper ? make_float2(px - v[i].x, py - v[i].y)
+                                       : make_float2(v[i].x + px, v[i].y + py);
+                v[i] = cmul(d, twl[st]);
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < R; ++i) acc[i] += v[i].x * v[i].x + v[i].y * v[i].y;
+    }
+    const int k2 = (int)(__brev((unsigned)lane) >> 27);
+#pragma unroll
+    for (int i = 0; i < R; ++i) {
+        const int k1 = (int)(__brev((unsigned)i) >> (32 - LOG2R));
+        acc_sh[warp][k1 + R * k2] = acc[i];
+    }
+    __syncthreads();
+    constexpr float invN = 1.0f / (float)N;             // a power of two: exact
+    for (int b = threadIdx.x; b <= HALF; b += blockDim.x) {
+        float s = 0.f;
+        for (int w = 0; w < kWarpEnergyWarps; ++w) s += acc_sh[w][b];
+        if (b > 0 && b < HALF) {
+            float m = 0.f;
+            for (int w = 0; w < kWarpEnergyWarps; ++w) m += acc_sh[w][N - b];
+            s += m;
+        }
+        bins[b] = s * invN;
+    }
+    __syncthreads();
+    const int n_bins = HALF + 1;
+    for (int b = warp; b < n_bands; b += kWarpEnergyWarps) {
+        const int lo = (n_bins * b) / n_bands, hi = (n_bins * (b + 1)) / n_bands;
+        float s = 0.f;
+        for (int k = lo + lane; k < hi; k += 32) s += bins[k];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if (lane == 0) {
+            bands[b] = s;
+            band_out[(int64_t)tau * n_bands + b] = s;
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float e = 0.f;
+        for (int b = 0; b < n_bands; ++b) e += bands[b];
+        seg_out[tau] = sqrtf(e);
+    }
+}
+
 }  // namespace
 
 extern "C" echo_status echo_audio_energy(const float *audio, int64_t n_samples, int32_t T,
@@ -140,11 +306,28 @@ extern "C" echo_status echo_audio_energy(const float *audio, int64_t n_samples, 
 
     const int seg_len = (int)(n_samples / T);
     const int n_frames = seg_len < n_fft ? 1 : (seg_len - n_fft) / hop + 1;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (n_fft <= 512 && n_bands <= 64) {   // the warp-per-frame-pair kernel
+        LaunchScope ls(ECHO_K_ENERGY, T, n_frames, n_fft, st);
+        const int R = n_fft / 32;
+        if (R == 2)
+            segment_energy_warp_kernel<2><<<T, kWarpEnergyWarps * 32, 0, st>>>(
+                audio, seg_len, hop, n_frames, n_bands, band_energy, seg_energy);
+        else if (R == 4)
+            segment_energy_warp_kernel<4><<<T, kWarpEnergyWarps * 32, 0, st>>>(
+                audio, seg_len, hop, n_frames, n_bands, band_energy, seg_energy);
+        else if (R == 8)
+            segment_energy_warp_kernel<8><<<T, kWarpEnergyWarps * 32, 0, st>>>(
+                audio, seg_len, hop, n_frames, n_bands, band_energy, seg_energy);
+        else
+            segment_energy_warp_kernel<16><<<T, kWarpEnergyWarps * 32, 0, st>>>(
+                audio, seg_len, hop, n_frames, n_bands, band_energy, seg_energy);
+        return last_launch_status();
+    }
     int log2n = 0;
     while ((1 << log2n) < n_fft) ++log2n;
     const size_t smem = sizeof(float2) * (size_t)(n_fft / 2 + kGroups * n_fft) +
                         sizeof(float) * (size_t)kGroups * n_bins;
-    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     if (smem > 48 * 1024 &&
         cudaFuncSetAttribute(segment_energy_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem) != cudaSuccess)
