@@ -72,7 +72,10 @@ def test_audio_energy(ec, name, profile):
 def test_audio_energy_short_segments_and_other_fft(ec):
     g = np.random.default_rng(0)
     a = g.standard_normal(3000).astype(F32)
-    for T, n_fft, hop, nb in ((10, 512, 160, 8), (3, 256, 100, 5), (2, 1024, 333, 3)):
+    # 64 .. 512 take the warp kernel (two frames per complex FFT), 1024 the
+    # shared-memory kernel; odd frame counts leave a lone last frame
+    for T, n_fft, hop, nb in ((10, 512, 160, 8), (3, 256, 100, 5), (2, 1024, 333, 3),
+                              (5, 64, 20, 4), (2, 128, 50, 3), (1, 512, 160, 64)):
         band, seg = ec.echo_audio_energy(f32(a), T, n_fft, hop, nb)
         ob, oe = oracle.energy.audio_energy(a, T, n_fft, hop, nb)
         assert np.allclose(seg.cpu().numpy(), oe, rtol=1e-5, atol=0)
@@ -316,6 +319,13 @@ ATTN_CASES = [
     (128, 64, 4, 128),
     (130, 672, 3, 128),
     (64, 7800, 2, 64),
+    # key sets up to 4096 take the persistent kernel (items chained per SM)
+    (6552, 672, 40, 128),    # cross-attention of the 32760-token block: 1040 items, 96-key blocks
+    (3000, 160, 16, 64),     # 192 items (some CTAs take two), 96-key blocks with a masked tail
+    (1000, 64, 4, 128),      # 64-key blocks
+    (300, 32, 3, 64),        # 32-key blocks
+    (300, 4096, 2, 64),      # the largest key set of the persistent kernel
+    (300, 4097, 2, 64),      # one key more: the one-shot kernel
 ]
 
 
