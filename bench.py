@@ -142,6 +142,12 @@ def algorithmic_work(name, m, n, k, K, xbytes=2):
         # already in y (stored by the FFN-down epilogue); the row map once
         NT, D = m, n
         return None, (NT - K) * (3.0 * D + 4) + 4.0 * NT
+    if name == "merge_quant":
+        # every row once: an inactive row's codes and scale in, bf16 out; an
+        # active row's bf16 value and row max in, codes and scale out; the row
+        # map once
+        NT, D = m, n
+        return None, NT * (3.0 * D + 8) + 4.0 * K
     if name == "quant_scatter":
         return None, m * n * 3 + 8.0 * m
     if name == "layernorm_gather":

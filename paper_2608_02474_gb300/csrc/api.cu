@@ -171,7 +171,8 @@ extern "C" const char *echo_kernel_name(int32_t kind) {
         "segment_energy_fft", "drift_score",  "topk_select",  "rowmap",
         "layernorm_gather",   "gemm_tcgen05", "attention",    "quant_scatter",
         "dequant_gather",     "dequant_merge", "step_delta",   "uniform_select",
-        "ref_scan",           "ref_alloc",     "ref_store",    "cache_copy"};
+        "ref_scan",           "ref_alloc",     "ref_store",    "cache_copy",
+        "merge_quant"};
     if (kind < 0 || kind >= ECHO_K_COUNT) return "unknown";
     return names[kind];
 }

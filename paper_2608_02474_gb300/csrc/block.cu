@@ -16,8 +16,8 @@
 //   GEMM        y[idx] = u W2^T + b2 + h2               (bf16, stored at the
 //               active tokens' rows of y; the epilogue also folds max |y| per
 //               row for the quantiser)
-//   merge       y = reconstructed cache at every other row
-//   quant       cache[idx] = Q(y[idx])                  (one pass)
+//   merge+quant y = reconstructed cache at every other row, and
+//               cache[idx] = Q(y[idx]), in one pass over the rows
 #include "common.cuh"
 #include "internal.h"
 
@@ -171,12 +171,10 @@ extern "C" echo_status echo_block_step(const echo_block_weights *w, const echo_b
     s = run_active(w, d, x, idx, K, ws, L, st, y);
     if (s != ECHO_OK) return s;
     const int32_t *rowmap = reinterpret_cast<const int32_t *>(ws + L.rowmap);
-    // the merge fills the inactive rows from the cache; the quantiser reads the
-    // active rows of y and writes the active rows of the cache: no overlap
-    launch_dequant_merge(cache_q, cache_scale, rowmap, nullptr, NT, d.D, y, st);
-    if (K > 0)
-        launch_quant_amax(y, reinterpret_cast<const uint32_t *>(ws + L.amax), idx, K, d.D,
-                          cache_q, cache_scale, st);
+    // one pass over every row: an inactive row is reconstructed from the cache
+    // into y, an active row of y is quantised into the cache (disjoint rows)
+    launch_merge_quant(cache_q, cache_scale, rowmap, reinterpret_cast<const uint32_t *>(ws + L.amax),
+                       NT, d.D, K, y, st);
     return last_launch_status();
 }
 

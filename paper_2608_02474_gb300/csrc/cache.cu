@@ -88,63 +88,6 @@ quant_kernel(const ST *__restrict__ src, const int32_t *__restrict__ rows, int n
     }
 }
 
-// quant_kernel with the row's max |v| given (computed where the rows were
-// produced): one read of each row.  Same rules and the same bits.
-__global__ void __launch_bounds__(kQuantThreads)
-quant_amax_kernel(const __nv_bfloat16 *__restrict__ src, const uint32_t *__restrict__ amax_bits,
-                  const int32_t *__restrict__ rows, int n_rows, int D, int8_t *__restrict__ q,
-                  float *__restrict__ scale, int *err) {
-    const int lane = threadIdx.x & 31;
-    const int warps = blockDim.x >> 5;
-    const int C = D >> 3;
-    for (int j = blockIdx.x * warps + (threadIdx.x >> 5); j < n_rows; j += gridDim.x * warps) {
-        const int r = rows ? rows[j] : j;
-        const __nv_bfloat16 *s = src + (int64_t)r * D;   // the rows sit at their token positions
-        const uint32_t ab = amax_bits[j];
-        const float amax = __uint_as_float(ab);
-        int8_t *qr = q + (int64_t)r * D;
-        if (ab >= 0x7F800000u) {   // NaN or infinity in the row
-            for (int c = lane; c < C; c += 32) *reinterpret_cast<uint2 *>(qr + 8 * c) = make_uint2(0, 0);
-            if (lane == 0) {
-                scale[r] = ab > 0x7F800000u ? __int_as_float(0x7fc00000) : INFINITY;
-                echo_flag_error(err, ECHO_ERR_NONFINITE);
-            }
-            continue;
-        }
-        float sc = 0.f, inv = 0.f;
-        if (amax > 0.f) {
-            sc = __fdiv_rn(amax, 127.f);
-            inv = __fdiv_rn(127.f, amax);
-        }
-        // four 16-byte loads in flight per lane before any of them is used
-        for (int c0 = lane; c0 < C; c0 += 4 * 32) {
-            uint4 u[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int c = c0 + 32 * i;
-                u[i] = c < C ? __ldcs(reinterpret_cast<const uint4 *>(s + 8 * c)) : make_uint4(0, 0, 0, 0);
-            }
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int c = c0 + 32 * i;
-                if (c >= C) break;
-                float f[8];
-                unpack8_bf16(u[i], f);
-                uint32_t w[2] = {0u, 0u};
-#pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    float t = rintf(__fmul_rn(f[k], inv));
-                    t = fminf(fmaxf(t, -127.f), 127.f);
-                    const uint32_t b = (uint32_t)(uint8_t)(int8_t)(int)t;
-                    w[k >> 2] |= b << (8 * (k & 3));
-                }
-                *reinterpret_cast<uint2 *>(qr + 8 * c) = make_uint2(w[0], w[1]);
-            }
-        }
-        if (lane == 0) scale[r] = sc;
-    }
-}
-
 ECHO_DEV void dequant16(const int4 &qv, float s, float *f) {
     const int8_t *b = reinterpret_cast<const int8_t *>(&qv);
 #pragma unroll
@@ -220,6 +163,64 @@ dequant_merge_kernel(const int8_t *__restrict__ q, const float *__restrict__ sca
     }
 }
 
+// The merge and the int8 write of the active rows in one pass over every row
+// (Sec. 3.3 mask fusion, Sec. 3.4 cache write): 16 elements per thread.  A row
+// with rowmap[i] < 0 is reconstructed from the cache into y (bf16(q s)); an
+// active row, which the FFN-down epilogue already stored in y together with
+// its max |v| (amax_bits[rowmap[i]], fp32 bits), is quantised into the cache
+// with the rules and bits of quant_kernel (the thread of the row's first 16
+// elements writes its scale).  Both kinds move 3 bytes per element.
+__global__ void __launch_bounds__(kVecThreads)
+merge_quant_kernel(int8_t *__restrict__ q, float *__restrict__ scale,
+                   const int32_t *__restrict__ rowmap, const uint32_t *__restrict__ amax_bits,
+                   int NT, int D, __nv_bfloat16 *__restrict__ y, int *err) {
+    const int C = D >> 4;
+    const int64_t total = (int64_t)NT * C;
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+         t += (int64_t)gridDim.x * blockDim.x) {
+        const int i = (int)(t / C), c = (int)(t % C);
+        const int pos = rowmap[i];
+        uint4 *o = reinterpret_cast<uint4 *>(y + (int64_t)i * D + 16 * c);
+        int4 *qr = reinterpret_cast<int4 *>(q + (int64_t)i * D + 16 * c);
+        if (pos < 0) {
+            const int4 qv = __ldcs(qr);
+            float f[16];
+            dequant16(qv, scale[i], f);
+            __stcs(o, pack8_bf16(f));
+            __stcs(o + 1, pack8_bf16(f + 8));
+            continue;
+        }
+        const uint32_t ab = amax_bits[pos];
+        if (ab >= 0x7F800000u) {   // NaN or infinity in the row
+            __stcs(qr, make_int4(0, 0, 0, 0));
+            if (c == 0) {
+                scale[i] = ab > 0x7F800000u ? __int_as_float(0x7fc00000) : INFINITY;
+                echo_flag_error(err, ECHO_ERR_NONFINITE);
+            }
+            continue;
+        }
+        const float amax = __uint_as_float(ab);
+        float sc = 0.f, inv = 0.f;
+        if (amax > 0.f) {
+            sc = __fdiv_rn(amax, 127.f);
+            inv = __fdiv_rn(127.f, amax);
+        }
+        const uint4 v0 = __ldcs(o), v1 = __ldcs(o + 1);
+        float f[16];
+        unpack8_bf16(v0, f);
+        unpack8_bf16(v1, f + 8);
+        uint32_t w[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+            float r = rintf(__fmul_rn(f[k], inv));
+            r = fminf(fmaxf(r, -127.f), 127.f);
+            w[k >> 2] |= (uint32_t)(uint8_t)(int8_t)(int)r << (8 * (k & 3));
+        }
+        __stcs(qr, make_int4((int)w[0], (int)w[1], (int)w[2], (int)w[3]));
+        if (c == 0) scale[i] = sc;
+    }
+}
+
 int grid_for(int64_t work, int threads) {
     int64_t g = (work + threads - 1) / threads;
     const int64_t cap = 152 * 32;
@@ -245,16 +246,6 @@ void launch_quant(const void *src, echo_dtype st_t, const int32_t *rows, int32_t
     else
         quant_kernel<float><<<grid, kQuantThreads, 0, st>>>(static_cast<const float *>(src), rows,
                                                             n_rows, D, q, scale, err);
-}
-
-void launch_quant_amax(const void *src, const uint32_t *amax, const int32_t *rows, int32_t n_rows,
-                       int32_t D, int8_t *q, float *scale, cudaStream_t st) {
-    if (n_rows <= 0) return;
-    const int grid = grid_for((int64_t)n_rows * 32, kQuantThreads);
-    LaunchScope ls(ECHO_K_QUANT, n_rows, D, 0, st);
-    quant_amax_kernel<<<grid, kQuantThreads, 0, st>>>(static_cast<const __nv_bfloat16 *>(src), amax,
-                                                      rows, n_rows, D, q, scale,
-                                                      device_error_ptr());
 }
 
 void launch_dequant(const int8_t *q, const float *scale, const int32_t *rows, int32_t n_rows,
@@ -285,6 +276,15 @@ void launch_dequant_merge(const int8_t *q, const float *scale, const int32_t *ro
     dequant_merge_kernel<<<grid, kVecThreads, 0, st>>>(
         q, scale, rowmap, static_cast<const __nv_bfloat16 *>(y_act), NT, D,
         static_cast<__nv_bfloat16 *>(y));
+}
+
+void launch_merge_quant(int8_t *q, float *scale, const int32_t *rowmap, const uint32_t *amax,
+                        int32_t NT, int32_t D, int32_t K, void *y, cudaStream_t st) {
+    const int grid = grid_for((int64_t)NT * (D / 16), kVecThreads);
+    LaunchScope ls(ECHO_K_MERGE_QUANT, NT, D, K, st);
+    merge_quant_kernel<<<grid, kVecThreads, 0, st>>>(q, scale, rowmap, amax, NT, D,
+                                                     static_cast<__nv_bfloat16 *>(y),
+                                                     device_error_ptr());
 }
 
 }  // namespace echo

@@ -66,15 +66,16 @@ echo_status launch_attention(const void *Q, int64_t ldq, const void *K, const vo
 // cache.cu
 void launch_quant(const void *src, echo_dtype st_t, const int32_t *rows, int32_t n_rows,
                   int32_t D, int8_t *q, float *scale, cudaStream_t st);
-// int8 quantisation of bf16 rows whose max |v| is already known (fp32 bits):
-// row j is read from src row rows[j] and written to cache row rows[j]
-void launch_quant_amax(const void *src, const uint32_t *amax, const int32_t *rows, int32_t n_rows,
-                       int32_t D, int8_t *q, float *scale, cudaStream_t st);
 void launch_dequant(const int8_t *q, const float *scale, const int32_t *rows, int32_t n_rows,
                     int32_t D, void *dst, echo_dtype dt, cudaStream_t st);
 void launch_rowmap(const int32_t *idx, int32_t K, int32_t NT, int32_t *rowmap, cudaStream_t st);
 void launch_dequant_merge(const int8_t *q, const float *scale, const int32_t *rowmap,
                           const void *y_act, int32_t NT, int32_t D, void *y, cudaStream_t st);
+// y[i] = bf16(q[i] s[i]) for rowmap[i] < 0; every other row of y (already the
+// fresh block output, max |y| per row in amax[rowmap[i]]) is quantised into
+// q[i], s[i]: the merge and the int8 write of the block step in one pass
+void launch_merge_quant(int8_t *q, float *scale, const int32_t *rowmap, const uint32_t *amax,
+                        int32_t NT, int32_t D, int32_t K, void *y, cudaStream_t st);
 
 // refcache.cu: cache forms other than plain int8 (and int8 through the same calls)
 echo_status cache_check(const echo_cache *c);

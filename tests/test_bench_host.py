@@ -25,6 +25,9 @@ def test_algorithmic_work_of_the_contractions_and_bandwidth_kernels():
     # merge: the inactive rows (codes in, bf16 out, scale) and the row map
     assert bench.algorithmic_work("dequant_merge", NT, D, 0, K) == (
         None, (NT - K) * (3.0 * D + 4) + 4.0 * NT)
+    # merge + int8 write: 3 bytes per element of every row, the scale or row
+    # max and the row map per row, the active rows' scales out
+    assert bench.algorithmic_work("merge_quant", NT, D, K, K) == (None, NT * (3.0 * D + 8) + 4.0 * K)
     # the all-latent layernorm also writes the K active rows' copy; a gathered
     # (K-row) layernorm of fp32 input does not
     assert bench.algorithmic_work("layernorm_gather", NT, D, 2, K) == (

@@ -82,7 +82,7 @@ def test_profile_report_from_env(ec, tmp_path, monkeypatch):
     rep = st.profile_report()
     ec.echo_profile_enable(False)
     names = {k.split("[")[0] for k in rep}
-    assert {"gemm_tcgen05", "attention", "drift_score", "topk_select", "dequant_merge"} <= names
+    assert {"gemm_tcgen05", "attention", "drift_score", "topk_select", "merge_quant"} <= names
     assert json.loads(out.read_text()) == json.loads(json.dumps(rep))
     assert all(v["launches"] > 0 and v["ms"] >= 0 for v in rep.values())
 
