@@ -132,17 +132,26 @@ def _run_trajectory(ec, w, steps, layers, profile="speech", el_rows=256):
     for t, l, x, q, s, r in rec:
         g_idx, y, qd, sd = gpu_layer(ec, blks[l], w, x, q, s, e32, (w.ratio_num, w.ratio_den),
                                      full=t == 0)
-        tag = f"{w.name} t={t} l={l}"
-        assert np.array_equal(g_idx, r.idx)
-        g = y.float().cpu().numpy()
-        mx, mean = normwise_rel(g[r.idx], r.y_act)
-        assert mx <= 2e-2 and mean <= 5e-3, (tag, mx, mean)
-        j = np.arange(len(r.idx))
-        if len(j) > el_rows:
-            j = _sample_rows(j, r.scores[r.idx] if t else np.zeros(len(j), F32), n=el_rows // 2)
-        emu = M.block_active(x, r.idx[j], Ws[l], cond, w.H)
+        check_step(ec, w, Ws[l], cond, x, q, s, r, g_idx, y, qd, sd, f"{w.name} t={t} l={l}",
+                   el_rows)
+
+
+def check_step(ec, w, W, cond, x, q, s, r, g_idx, y, qd, sd, tag, el_rows=256):
+    """One layer step against the oracle's result r on the same inputs: the
+    indices, every active row at the normwise and mean bars, up to `el_rows`
+    active rows (half at random, half of highest score) against the ideal bf16
+    model element-wise, the inactive rows and the cache write."""
+    assert np.array_equal(g_idx, r.idx)
+    g = y.float().cpu().numpy()
+    mx, mean = normwise_rel(g[r.idx], r.y_act)
+    assert mx <= 2e-2 and mean <= 5e-3, (tag, mx, mean)
+    j = np.arange(len(r.idx))
+    if len(j) > el_rows:
+        j = _sample_rows(j, r.scores[r.idx], n=el_rows // 2)
+    if len(j):
+        emu = M.block_active(x, r.idx[j], W, cond, w.H)
         check_active(g[r.idx[j]], r.y_act[j], emu, tag)
-        check_cache_and_inactive(ec, w, r.idx, q, s, g, y, qd.cpu().numpy(), sd.cpu().numpy())
+    check_cache_and_inactive(ec, w, r.idx, q, s, g, y, qd.cpu().numpy(), sd.cpu().numpy())
 
 
 def test_tiny_every_step(ec):

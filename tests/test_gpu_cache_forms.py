@@ -148,7 +148,7 @@ def _device_cache_from(ec, o, w):
 
 @pytest.mark.parametrize("kind", ["bf16", "ref"])
 def test_layer_step_with_cache_forms_teacher_forced(ec, kind):
-    from test_gpu_block import rel_err
+    from bf16_model import normwise_rel as rel_err
     w = TINY_256
     audio = G.audio(w)
     _, e = oracle.energy.audio_energy(audio, w.T)
@@ -195,7 +195,7 @@ def test_ref_cache_block_full_size_sampled(ec):
     64 sampled active rows are held to the normwise bars, and the cache write
     equals echo_cache_write of the rows the step returned."""
     from synth import WAN_BLOCK_32760 as w
-    from test_gpu_block import rel_err
+    from bf16_model import normwise_rel as rel_err
     audio = G.audio(w)
     _, e = oracle.energy.audio_energy(audio, w.T)
     e32 = e.astype(F32)

@@ -123,7 +123,7 @@ def _adaptive_trajectory(w, steps, layers, sch):
 @pytest.mark.parametrize("w,steps", [(TINY_256, TINY_256.steps), (STACK4_7800, 4)],
                          ids=["tiny_256", "stack4_7800"])
 def test_adaptive_loop_teacher_forced(ec, w, steps):
-    from test_gpu_block import check_layer, gpu_layer
+    from test_gpu_block import check_step, gpu_layer
     sch = S.Schedule(w.NT)
     Ws, cond, e32, rec = _adaptive_trajectory(w, steps, w.layers, sch)
     last = w.layers - 1
@@ -143,7 +143,7 @@ def test_adaptive_loop_teacher_forced(ec, w, steps):
     for t, l, x, q, s, r in rec:
         ratio = (w.ratio_num, w.ratio_den) if t == 0 else (g_budget[t - 1], w.NT)
         g_idx, y, qd, sd = gpu_layer(ec, blks[l], w, x, q, s, e32, ratio, full=t == 0)
-        check_layer(ec, w, r, q, s, g_idx, y, qd, sd)
+        check_step(ec, w, Ws[l], cond, x, q, s, r, g_idx, y, qd, sd, f"adaptive {w.name} t={t} l={l}")
 
 
 def _stack(ec, w):
