@@ -5,6 +5,7 @@
     python -m paper_2608_02474_gb300.kernel_bench --kernel drift --T 21 --N 1560 --D 5120
     python -m paper_2608_02474_gb300.kernel_bench --kernel merge --T 21 --N 1560 --D 5120 --K 6552
     python -m paper_2608_02474_gb300.kernel_bench --kernel step_delta --T 21 --N 1560 --D 5120
+    python -m paper_2608_02474_gb300.kernel_bench --kernel block --T 21 --N 1560 --D 5120 --K 6552
 
 Inputs are seeded random device tensors of the right shapes (values do not
 change the work of these kernels).  Prints the mean time per launch over
@@ -25,7 +26,7 @@ def make_parser() -> argparse.ArgumentParser:
     ap = argparse.ArgumentParser()
     ap.add_argument("--kernel", required=True,
                     choices=["gemm", "attention", "drift", "select", "merge", "quant", "layernorm",
-                             "energy", "step_delta", "ref_write"])
+                             "energy", "step_delta", "ref_write", "block"])
     ap.add_argument("--M", type=int, default=6552)
     ap.add_argument("--N", type=int, default=5120)
     ap.add_argument("--K", type=int, default=5120)
@@ -38,6 +39,8 @@ def make_parser() -> argparse.ArgumentParser:
     ap.add_argument("--rows", type=int, default=0, help="layernorm: gather this many rows")
     ap.add_argument("--f32", action="store_true", help="layernorm: fp32 input")
     ap.add_argument("--samples", type=int, default=80960, help="energy: audio samples")
+    ap.add_argument("--F", type=int, default=13824, help="block: FFN width")
+    ap.add_argument("--Lc", type=int, default=672, help="block: audio condition tokens")
     ap.add_argument("--iters", type=int, default=3)
     ap.add_argument("--warmup", type=int, default=1)
     return ap
@@ -124,6 +127,29 @@ def main():
         ws = torch.empty(cache.write_workspace_size(a.K), dtype=torch.uint8, device=dev)
         run = lambda: cache.write(src, rows, workspace=ws)
         work, unit = a.K * (3.0 * D + 8), "GB/s"
+    elif a.kernel == "block":
+        # one cached layer step (echo_block_step) on K of T*N tokens with
+        # random weights: every kernel of the block, for captures of any of them
+        NT, D, K = a.T * a.N, a.D, a.K
+        W = {}
+        for nm in ("q", "k", "v", "o", "qc", "kc", "vc", "oc"):
+            W["W" + nm] = (rn(D, D) * 0.02).to(torch.bfloat16)
+            W["b" + nm] = (rn(D) * 0.02).to(torch.bfloat16)
+        W["W1"], W["b1"] = (rn(a.F, D) * 0.02).to(torch.bfloat16), (rn(a.F) * 0.02).to(torch.bfloat16)
+        W["W2"], W["b2"] = (rn(D, a.F) * 0.02).to(torch.bfloat16), (rn(D) * 0.02).to(torch.bfloat16)
+        blk = ec.DeviceBlock.from_host(W, rn(a.Lc, D).to(torch.bfloat16), device=dev)
+        del W
+        dims = ec.BlockDims(a.T, a.N, D, a.H, a.d, a.F, a.Lc)
+        x = rn(NT, D).to(torch.bfloat16)
+        q = torch.randint(-127, 128, (NT, D), generator=g, device=dev, dtype=torch.int8)
+        s = torch.rand(NT, generator=g, device=dev) * 0.05
+        idx = torch.sort(torch.randperm(NT, generator=g, device=dev)[:K]).values.to(torch.int32)
+        y = torch.empty(NT, D, dtype=torch.bfloat16, device=dev)
+        ws = torch.empty(ec.echo_workspace_size(dims, K), dtype=torch.uint8, device=dev)
+        run = lambda: ec.echo_block_step(blk, dims, x, idx, K, q, s, y=y, workspace=ws)
+        work = (2.0 * NT * D * 2 * D + 4 * 2.0 * K * D * D + 4.0 * K * NT * D
+                + 4.0 * K * a.Lc * D + 2 * 2.0 * K * D * a.F)
+        unit = "TFLOP/s"
     elif a.kernel == "energy":
         audio = rn(a.samples)
         band = torch.empty(a.T, 8, dtype=torch.float32, device=dev)
