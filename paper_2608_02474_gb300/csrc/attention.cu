@@ -404,8 +404,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 // block is issued right after the last P V of the current one, so the tensor
 // cores keep working while the softmax warps run the epilogue.  Q is double
 // buffered: warp 3 (idle in the kernel above) copies the Q tiles of item k + 2
-// as soon as item k's epilogue has released its buffer; the epilogue stages O
-// through that item's finished Q buffer as above.  The key block BN (96 for the
+// as soon as item k's epilogue has released its buffer.  The epilogue stages O
+// in that item's finished Q buffer as above, and its global stores go out a few
+// at a time after each of the next item's first four softmax blocks.  The key block BN (96 for the
 // 672 audio tokens: 7 blocks, no padding) is chosen per launch to waste few
 // keys.  Ring positions, S/P/PV barrier phases and block counters run on
 // across items.
@@ -645,6 +646,41 @@ attn_items_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
         const uint32_t s_col = (uint32_t)(t * 128);
         const uint32_t o_col = O_COL + (uint32_t)(t * DH);
         const float sl2 = p.scale_log2;
+        constexpr int RB = DH * 2, CH = RB / 16;               // bytes and 16-byte chunks per row
+        constexpr int RPI = 32 / CH;                           // rows per warp-wide store
+        constexpr int N_ST = 32 / RPI;                         // warp-wide stores per item
+        // spread over the next item's first min(nb, 4) blocks, so that the
+        // buffer is released before the next item's last block: the Q of the
+        // item after next, which the MMA warp waits for there, needs it
+        const int spread = nb < 4 ? nb : 4;
+        const int st_per_block = (N_ST + spread - 1) / spread;
+        auto stage_of = [&](int k) {
+            return Qs + (k & 1) * C::QBUF_BYTES + t * C::Q_BYTES + quad * 32 * RB;
+        };
+        // Item k's O leaves its staging buffer in parts, a few warp-wide stores
+        // after each of the next item's first softmax blocks, so that the
+        // stores overlap that work instead of holding the warp at the item
+        // boundary; the buffer then goes back to the Q producer.
+        int pend_k = -1, pend_i = 0;
+        auto store_part = [&](int n) {
+            const uint8_t *stage = stage_of(pend_k);
+            const int row0 = item_tp(pend_k) * (TILES * BM) + t * BM + quad * 32;
+            const int col0 = item_h(pend_k) * DH;
+            const int end = pend_i + n < N_ST ? pend_i + n : N_ST;
+            for (; pend_i < end; ++pend_i) {
+                const int rr = pend_i * RPI + lane / CH, cc = lane % CH;
+                const uint4 v =
+                    *reinterpret_cast<const uint4 *>(stage + rr * RB + ((cc ^ (rr & (CH - 1))) * 16));
+                const int grow = row0 + rr;
+                if (grow < p.M)
+                    *reinterpret_cast<uint4 *>(p.O + (int64_t)grow * p.ldo + col0 + 8 * cc) = v;
+            }
+            if (pend_i == N_ST) {
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&q_empty[pend_k & 1]);   // done with the buffer
+                pend_k = -1;
+            }
+        };
         bool ok = true;
         for (int k = 0, f = 0; ok && k < n_items; ++k) {
             float m_used = -INFINITY, l = 0.f;
@@ -726,22 +762,27 @@ attn_items_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&p_full[t]);
+                if (pend_k >= 0) store_part(st_per_block);   // the previous item's O, in parts
             }
             if (!ok) break;
             ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[t], k & 1, abort_v, p.err));
             if (!ok) break;
             tc_fence_after();
             const float inv = 1.f / l;
-            constexpr int RB = DH * 2, CH = RB / 16;
-            uint8_t *stage = Qs + (k & 1) * C::QBUF_BYTES + t * C::Q_BYTES + quad * 32 * RB;
+            // every load of the row's O in flight before one wait
+            uint32_t o[DH / 32][32];
+#pragma unroll
+            for (int c = 0; c < DH / 32; ++c) tmem_ld32(tmem + lane_base + o_col + 32 * c, o[c]);
+            tmem_ld_wait();
+            // O of this item is out of tensor memory: the next item's first
+            // P V may overwrite it once this warp arrives on p_full next time
+            tc_fence_before();
+            uint8_t *stage = stage_of(k);
 #pragma unroll
             for (int c = 0; c < DH / 32; ++c) {
-                uint32_t o[32];
-                tmem_ld32(tmem + lane_base + o_col + 32 * c, o);
-                tmem_ld_wait();
                 float fo[32];
 #pragma unroll
-                for (int i = 0; i < 32; ++i) fo[i] = __uint_as_float(o[i]) * inv;
+                for (int i = 0; i < 32; ++i) fo[i] = __uint_as_float(o[c][i]) * inv;
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int cc = 4 * c + i;
@@ -749,25 +790,11 @@ attn_items_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
                         pack8_bf16(fo + 8 * i);
                 }
             }
-            // O of this item is out of tensor memory: the next item's first
-            // P V may overwrite it once this warp arrives on p_full next time
-            tc_fence_before();
             __syncwarp();
-            const int row0 = item_tp(k) * (TILES * BM) + t * BM + quad * 32;
-            const int col0 = item_h(k) * DH;
-            constexpr int RPI = 32 / CH;
-#pragma unroll
-            for (int kk = 0; kk < 32 / RPI; ++kk) {
-                const int rr = kk * RPI + lane / CH, cc = lane % CH;
-                const uint4 v =
-                    *reinterpret_cast<const uint4 *>(stage + rr * RB + ((cc ^ (rr & (CH - 1))) * 16));
-                const int grow = row0 + rr;
-                if (grow < p.M)
-                    *reinterpret_cast<uint4 *>(p.O + (int64_t)grow * p.ldo + col0 + 8 * cc) = v;
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&q_empty[k & 1]);   // this warp is done with the buffer
+            pend_k = k;
+            pend_i = 0;
         }
+        if (ok && pend_k >= 0) store_part(N_ST);
     }
     tc_fence_before();
     __syncthreads();
