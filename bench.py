@@ -66,6 +66,10 @@ def parse():
     ap.add_argument("--latents", default="iid", choices=["iid", "smooth"],
                     help="synthetic latents: i.i.d. (default) or spatially smooth rows "
                          "(AR(1) along each frame row, rho 0.95)")
+    ap.add_argument("--reuse-kv", action="store_true",
+                    help="keep every layer's K/V of all tokens on the device across steps and "
+                         "recompute, at layers >= 1, only the rows whose input changed (the "
+                         "outputs are bit for bit those without)")
     ap.add_argument("--graph", action="store_true",
                     help="replay each step (audio energy included) as a captured CUDA graph; "
                          "one host launch per step")
@@ -371,6 +375,7 @@ def workload_config(args, w, rnum, rden, K, world):
             "audio": args.profile, "parallelism": f"replicas{world}",
             "cache": args.cache, "selection": args.select,
             "latents": args.latents, "graph": bool(args.graph),
+            "reuse_kv": bool(getattr(args, "reuse_kv", False)),
             "l2": "inputs larger than L2 (x 335 MB, weights 702 MB per block)"}
 
 
@@ -562,7 +567,7 @@ def make_stack(args, w, blocks, dev):
     kinds = {"int8": ec.CACHE_INT8, "bf16": ec.CACHE_BF16, "ref": ec.CACHE_REF}
     return CachedStack(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc, blocks, device=dev,
                        cache_kind=kinds[args.cache], seg_len=args.seg_len or w.Wp, tau=args.tau,
-                       selection=args.select)
+                       selection=args.select, reuse_kv=bool(getattr(args, "reuse_kv", False)))
 
 
 def run_sweep(args, w, blocks, x0, xs, dev, rank, world):
@@ -693,8 +698,8 @@ def main():
     eager_step = one_step
     graph_launches = None
     if args.graph:
-        if rate is not None or args.select == "random":
-            raise SystemExit("--graph takes a fixed ratio and no random selection")
+        if rate is not None or args.select == "random" or args.reuse_kv:
+            raise SystemExit("--graph takes a fixed ratio, no random selection and no --reuse-kv")
         stack.set_audio(audio_d)
         stack.step(xs_d[0], rnum, rden)             # one-time kernel set-up outside capture
         ybufs = [torch.empty_like(xs_d[0]) for _ in range(2)]

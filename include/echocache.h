@@ -377,6 +377,44 @@ echo_status echo_block_step(const echo_block_weights *w, const echo_block_dims *
                             int8_t *cache_q, float *cache_scale, void *y,
                             void *workspace, size_t ws_bytes, echo_stream_t stream);
 
+/* echo_block_step with the K/V of every token kept in a caller-owned buffer
+ * across steps, recomputed only for the tokens whose layer input changed.
+ * Sec. 3.3 takes K and V from the complete latent set at every step; a token's
+ * K/V row is a function of that token's layer input alone (row-wise layer norm
+ * and a GEMM whose reduction order per output row is fixed), so a row whose
+ * input did not change since it was computed is reused bit for bit.  In a
+ * stack, a token's input to layer l >= 1 changes between two steps only if the
+ * token was refreshed at layer l - 1 in either of them (fresh value one step,
+ * the reconstruction from the int8 cache the next); layer 0's input changes
+ * everywhere.  The results equal echo_block_step's on the same x, bit for bit,
+ * as long as the rows passed cover every row of x that differs from the input
+ * kv was computed from.
+ *   kv       bf16 [NT, 2D], device, 16-byte aligned: row i holds K_i | V_i.
+ *   kv_valid 0: kv's contents are ignored; K/V of every row are computed from x
+ *            (as echo_block_step does) and left in kv.  Non-zero: kv holds K/V
+ *            of an earlier input of this layer that differs from x at most at
+ *            the rows rows_a[0..n_a) and rows_b[0..n_b); only those are
+ *            recomputed (a row in both lists, or twice in one, is computed
+ *            again, to the same bits).  rows_a, rows_b int32 device arrays,
+ *            16-byte aligned, entries < NT; NULL when empty.
+ *   With K = 0 the block is skipped (y = reconstructed cache) but kv is still
+ *   brought up to date.  Other arguments as for echo_block_step.
+ *   workspace >= echo_workspace_size_kv(dims, K, n_a + n_b) bytes, 256-byte
+ *   aligned.
+ * The caller owns kv (NT x 2D x 2 bytes per layer: 671 MB for the
+ * 32760-token, D 5120 block) and decides which rows changed.
+ * Errors: INVALID_ARG, SHAPE, WORKSPACE, CUDA; NONFINITE/TIMEOUT device flags. */
+echo_status echo_block_step_kv(const echo_block_weights *w, const echo_block_dims *dims,
+                               const void *x, const int32_t *idx, int32_t K, void *kv,
+                               int32_t kv_valid, const int32_t *rows_a, int32_t n_a,
+                               const int32_t *rows_b, int32_t n_b, int8_t *cache_q,
+                               float *cache_scale, void *y, void *workspace, size_t ws_bytes,
+                               echo_stream_t stream);
+
+/* Bytes of workspace echo_block_step_kv needs for up to K_max active tokens and
+ * up to n_rows_max recomputed rows (n_a + n_b); also enough with kv_valid = 0. */
+size_t echo_workspace_size_kv(const echo_block_dims *dims, int32_t K_max, int32_t n_rows_max);
+
 /* Sec. 3.4, int8 per-token symmetric quantisation:
  *   q[rows[j]], scale[rows[j]] = Q(src[j]) for j < n_rows (rows NULL: j),
  *   Q(v): a = max|v|; a == 0 -> s = 0, q = 0; else s = a / 127,

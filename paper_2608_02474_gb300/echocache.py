@@ -90,6 +90,9 @@ _SIGS = {
     "echo_precompute_cross_kv": (_i32, [_vp, _vp, _vp, _i32, _i32, _vp, _vp]),
     "echo_block_step": (_i32, [_c.POINTER(BlockWeightsC), _c.POINTER(BlockDims), _vp, _vp, _i32,
                                _vp, _vp, _vp, _vp, _sz, _vp]),
+    "echo_workspace_size_kv": (_sz, [_c.POINTER(BlockDims), _i32, _i32]),
+    "echo_block_step_kv": (_i32, [_c.POINTER(BlockWeightsC), _c.POINTER(BlockDims), _vp, _vp, _i32,
+                                  _vp, _i32, _vp, _i32, _vp, _i32, _vp, _vp, _vp, _vp, _sz, _vp]),
     "echo_cache_quant": (_i32, [_vp, _i32, _vp, _i32, _i32, _vp, _vp, _vp]),
     "echo_cache_dequant": (_i32, [_vp, _vp, _vp, _i32, _i32, _vp, _i32, _vp]),
     "echo_linear": (_i32, [_vp, _i64, _i32, _i32, _vp, _vp, _i32, _i32, _vp, _i32, _vp, _vp, _i64,
@@ -269,6 +272,28 @@ def echo_block_step(weights: "DeviceBlock", dims: BlockDims, x, idx, K: int, cac
         _c.byref(weights.cstruct), _c.byref(dims), _p(x), _p(idx) if K > 0 else None, K,
         _p(cache_q), _p(cache_scale), _p(y), _p(workspace),
         workspace.numel() * workspace.element_size(), _stream(stream)))
+    return y
+
+
+def echo_workspace_size_kv(dims: BlockDims, K_max: int, n_rows_max: int) -> int:
+    return int(lib().echo_workspace_size_kv(_c.byref(dims), int(K_max), int(n_rows_max)))
+
+
+def echo_block_step_kv(weights: "DeviceBlock", dims: BlockDims, x, idx, K: int, kv,
+                       kv_valid: bool, cache_q, cache_scale, rows_a=None, n_a: int = 0,
+                       rows_b=None, n_b: int = 0, y=None, workspace=None, stream=None):
+    """echo_block_step with K/V of every token kept in `kv` (bf16 [NT, 2D])
+    across calls; with kv_valid only the rows rows_a[:n_a] and rows_b[:n_b]
+    are recomputed (the rows whose layer input changed)."""
+    y = y if y is not None else torch.empty_like(x)
+    if workspace is None:
+        workspace = torch.empty(echo_workspace_size_kv(dims, K, n_a + n_b), dtype=torch.uint8,
+                                device=x.device)
+    _check("echo_block_step_kv", lib().echo_block_step_kv(
+        _c.byref(weights.cstruct), _c.byref(dims), _p(x), _p(idx) if K > 0 else None, K,
+        _p(kv), 1 if kv_valid else 0, _p(rows_a) if n_a > 0 else None, n_a,
+        _p(rows_b) if n_b > 0 else None, n_b, _p(cache_q), _p(cache_scale), _p(y),
+        _p(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
     return y
 
 

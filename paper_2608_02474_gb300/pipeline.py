@@ -73,14 +73,21 @@ class CachedStack:
                  blocks: list, device="cuda", lam: float = 0.1, xi: float = 1e-6,
                  mode: int = ec.MODE_ENERGY_DRIFT, cache_kind: int = ec.CACHE_INT8,
                  R_cap: int | None = None, seg_len: int = 1, tau: float = 0.9,
-                 selection: str = "energy", seed: int = 0):
+                 selection: str = "energy", seed: int = 0, reuse_kv: bool = False):
         """cache_kind: ec.CACHE_INT8 (plain int8), ec.CACHE_BF16 (full
         precision) or ec.CACHE_REF (reference plus int8 residual, Sec. 3.4,
         with R_cap, seg_len and tau).  selection: "energy" (the energy-guided
         anchors of Sec. 3.3), or the ablations "uniform" and "random" (keys
-        drawn on the device from a generator seeded with `seed`)."""
+        drawn on the device from a generator seeded with `seed`).
+        reuse_kv (int8 cache only): keep every layer's K/V of all tokens on the
+        device (NT x 2D bf16 per layer) and recompute, at layers >= 1, only the
+        rows whose input changed: the tokens refreshed at the layer below in
+        this step or the step before (echo_block_step_kv).  The outputs are
+        bit for bit those without reuse."""
         if selection not in ("energy", "uniform", "random"):
             raise ValueError(f"unknown selection {selection!r}")
+        if reuse_kv and cache_kind != ec.CACHE_INT8:
+            raise ValueError("reuse_kv needs the int8 cache form")
         self.T, self.N, self.D = T, N, D
         self.NT = T * N
         self.dims = ec.BlockDims(T, N, D, H, d, F, Lc)
@@ -98,6 +105,19 @@ class CachedStack:
             self.caches = [ec.DeviceCache(cache_kind, self.NT, D, R_cap=R_cap, seg_len=seg_len,
                                           tau=tau, device=dev) for _ in range(L)]
             ws = ec.echo_block_step_cache_workspace_size(self.dims, self.NT, self.caches[0])
+        self.reuse_kv = reuse_kv
+        if reuse_kv:
+            # K/V of every token per layer; the active rows of every layer at
+            # the last two steps (slot t & 1), with their counts (NT: a full
+            # step, after which the next step recomputes every row)
+            ws = ec.echo_workspace_size_kv(self.dims, self.NT, self.NT)
+            self.kv = [torch.empty(self.NT, 2 * D, dtype=torch.bfloat16, device=dev)
+                       for _ in range(L)]
+            self._act = [[torch.empty(self.NT, dtype=torch.int32, device=dev) for _ in range(2)]
+                         for _ in range(L)]
+            self._act_K = [[self.NT, self.NT] for _ in range(L)]
+            self._kv_ok = [False] * L
+            self._t = 0
         self.ws = torch.empty(ws, dtype=torch.uint8, device=dev)
         self.keys = torch.empty(self.NT, dtype=torch.float32, device=dev)
         self.gen = torch.Generator(device=dev).manual_seed(seed)
@@ -171,6 +191,8 @@ class CachedStack:
             self._in_use, self._pending = self._pending, None
         cur = self._layers(x, ratio_num, ratio_den, full, keep_scores, out)
         self._seg_free[self._in_use].record(main)   # set_audio may now overwrite it
+        if self.reuse_kv:
+            self._t += 1
         return cur
 
     def _layers(self, x, ratio_num, ratio_den, full, keep_scores, out):
@@ -202,7 +224,9 @@ class CachedStack:
                                                  scores=self.scores if keep_scores else None,
                                                  workspace=self.sel_ws)
             dst = out if (l == last and out is not None) else self.y[l % 2]
-            if self.caches is None:
+            if self.reuse_kv:
+                self._block_step_kv(l, blk, cur, idx, K, dst)
+            elif self.caches is None:
                 ec.echo_block_step(blk, self.dims, cur, idx, K, self.cache_q[l], self.cache_s[l],
                                    y=dst, workspace=self.ws)
             else:
@@ -213,6 +237,25 @@ class CachedStack:
                 hook("post", l, cur, idx, K, dst)
             cur = dst
         return cur
+
+    def _block_step_kv(self, l, blk, x, idx, K, dst):
+        """Layer l's block step with its K/V kept across steps (reuse_kv)."""
+        t, NT = self._t, self.NT
+        valid, ra, na, rb, nb = False, None, 0, None, 0
+        if l > 0 and self._kv_ok[l]:
+            na, nb = self._act_K[l - 1][t & 1], self._act_K[l - 1][(t - 1) & 1]
+            if na + nb < NT:
+                valid = True
+                ra, rb = self._act[l - 1][t & 1], self._act[l - 1][(t - 1) & 1]
+        if not valid:
+            na = nb = 0
+        ec.echo_block_step_kv(blk, self.dims, x, idx, K, self.kv[l], valid, self.cache_q[l],
+                              self.cache_s[l], ra, na, rb, nb, y=dst, workspace=self.ws)
+        self._kv_ok[l] = True
+        if l + 1 < len(self.blocks):      # the next layer's changed rows
+            if 0 < K < NT:
+                self._act[l][t & 1][:K].copy_(idx[:K])
+            self._act_K[l][t & 1] = K if K < NT else NT
 
     def capture_step(self, x: torch.Tensor, ratio_num: int, ratio_den: int,
                      out: torch.Tensor | None = None, audio: torch.Tensor | None = None,
@@ -227,6 +270,8 @@ class CachedStack:
         that every kernel's one-time set-up is done."""
         if self.selection == "random":
             raise ValueError("random selection cannot be captured")
+        if self.reuse_kv:
+            raise ValueError("reuse_kv steps depend on the steps before them and cannot be captured")
         dev = self.seg.device
         self.wait_audio()
         if self._pending is not None:
@@ -255,6 +300,9 @@ class CachedStack:
             raise ValueError("cache state does not match this stack")
         if len(state["layers"]) != len(self.blocks):
             raise ValueError("cache state has a different number of layers")
+        if self.reuse_kv:   # the kept K/V belong to the old state
+            self._kv_ok = [False] * len(self.blocks)
+            self._act_K = [[self.NT, self.NT] for _ in self.blocks]
         for l, layer in enumerate(state["layers"]):
             if self.caches is None:
                 self.cache_q[l].copy_(layer["q"])

@@ -98,6 +98,38 @@ def test_block_step_argument_checks(ec):
     assert call(w_=ec.BlockWeightsC(*([FAKE] * 14 + [0]))) == 1     # null KVc
 
 
+def test_block_step_kv_argument_checks(ec):
+    """echo_block_step_kv: every check answers before anything is enqueued."""
+    L = ec.lib()
+    dims = ec.BlockDims(4, 64, 128, 2, 64, 512, 32)
+    w = ec.BlockWeightsC(*([FAKE] * 15))
+    ws = ec.echo_workspace_size_kv(dims, 64, 40)
+    assert ws > 0
+    call = lambda K=64, kv=FAKE, valid=1, ra=FAKE, na=20, rb=FAKE, nb=20, wsb=ws: L.echo_block_step_kv(
+        ctypes.byref(w), ctypes.byref(dims), _vp(FAKE), _vp(FAKE), K, _vp(kv), valid, _vp(ra), na,
+        _vp(rb), nb, _vp(FAKE), _vp(FAKE), _vp(FAKE), _vp(FAKE), wsb, None)
+    assert call(kv=0) == 1                       # no K/V buffer
+    assert call(kv=FAKE + 8) == 1                # misaligned K/V buffer
+    assert call(na=-1) == 2
+    assert call(ra=0) == 1                       # rows listed but no list
+    assert call(ra=FAKE + 4) == 1
+    assert call(K=257) == 2
+    assert call(wsb=4096) == 3                   # far below 64 active, 40 recomputed rows
+    # more rows need more workspace; kv_valid = 0 ignores the lists
+    assert ec.echo_workspace_size_kv(dims, 64, 41) >= ws
+    assert call(valid=0, ra=0, na=-5, wsb=ec.echo_workspace_size_kv(dims, 64, 0) - 1) == 3
+
+
+def test_workspace_size_kv_leaves_kv_to_the_caller(ec):
+    dims = ec.BlockDims(21, 1560, 5120, 40, 128, 13824, 672)
+    NT, D = 32760, 5120
+    plain = ec.echo_workspace_size(dims, 6552)
+    kept = ec.echo_workspace_size_kv(dims, 6552, NT)
+    # the all-token K/V (NT x 2D bf16) lives in the caller's buffer instead
+    assert plain - kept >= 4 * NT * D - 4 * NT - 4096
+    assert ec.echo_workspace_size_kv(dims, 6552, 13104) <= kept
+
+
 def test_workspace_size_grows_with_K(ec):
     dims = ec.BlockDims(21, 1560, 5120, 40, 128, 13824, 672)
     a, b = ec.echo_workspace_size(dims, 0), ec.echo_workspace_size(dims, 6552)
