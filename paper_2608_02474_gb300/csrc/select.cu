@@ -8,7 +8,8 @@
 //   16..1), with explicit round-to-nearest intrinsics so nothing is contracted.
 // topk_kernel: one CTA radix-selects the K-th largest 32-bit key (11/11/10-bit
 //   digits), then compacts in index order, taking keys equal to the threshold
-//   from the lowest index up.
+//   from the lowest index up.  Keys are read four at a time (16-byte loads,
+//   several in flight per thread): the kernel is bound by load latency.
 #include <mutex>
 
 #include "common.cuh"
@@ -207,11 +208,38 @@ topk_kernel(const float *__restrict__ scores, int NT, int K, int keys_in_smem,
     }
     if (K <= 0) return;
 
-    if (keys_in_smem)
-        for (int i = tid; i < NT; i += blockDim.x) skeys[i] = order_key(scores[i]);
+    // keys of elements i .. i + 3 (i a multiple of 4); those at or past NT are
+    // 0, below every key of a finite score
+    auto gkeys4 = [&](int i) -> uint4 {
+        if (i + 3 < NT) {
+            const float4 v = __ldg(reinterpret_cast<const float4 *>(scores + i));
+            return make_uint4(order_key(v.x), order_key(v.y), order_key(v.z), order_key(v.w));
+        }
+        uint32_t k[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) k[c] = i + c < NT ? order_key(scores[i + c]) : 0u;
+        return make_uint4(k[0], k[1], k[2], k[3]);
+    };
+    const int stride4 = blockDim.x * 4;
+    if (keys_in_smem) {
+        // eight 16-byte loads in flight per thread
+        for (int b = tid * 4; b < NT; b += stride4 * 8) {
+            uint4 v[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int i = b + u * stride4;
+                if (i < NT) v[u] = gkeys4(i);
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int i = b + u * stride4;
+                if (i < NT) *reinterpret_cast<uint4 *>(skeys + i) = v[u];
+            }
+        }
+    }
     __syncthreads();
-    auto key_at = [&](int i) -> uint32_t {
-        return keys_in_smem ? skeys[i] : order_key(scores[i]);
+    auto keys4 = [&](int i) -> uint4 {
+        return keys_in_smem ? *reinterpret_cast<const uint4 *>(skeys + i) : gkeys4(i);
     };
 
     uint32_t prefix = 0, pmask = 0;
@@ -223,9 +251,22 @@ topk_kernel(const float *__restrict__ scores, int NT, int K, int keys_in_smem,
         const int nb = 1 << widths[pass];
         for (int b = tid; b < 2048; b += blockDim.x) hist[b] = 0;
         __syncthreads();
-        for (int i = tid; i < NT; i += blockDim.x) {
-            const uint32_t k = key_at(i);
-            if ((k & pmask) == prefix) atomicAdd(&hist[(k >> sh) & (nb - 1)], 1);
+        for (int b = tid * 4; b < NT; b += stride4 * 4) {
+            uint4 v[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int i = b + u * stride4;
+                v[u] = i < NT ? keys4(i) : make_uint4(0, 0, 0, 0);
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int i = b + u * stride4;
+                const uint32_t k[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+                    if (i + c < NT && (k[c] & pmask) == prefix)
+                        atomicAdd(&hist[(k[c] >> sh) & (nb - 1)], 1);
+            }
         }
         __syncthreads();
         // thread t covers the two bins hi = nb-1-2t and lo = hi-1 (descending)
@@ -258,14 +299,16 @@ topk_kernel(const float *__restrict__ scores, int NT, int K, int keys_in_smem,
     for (int base = 0; base < NT; base += tile) {
         bool gt[kTopkItems], eq[kTopkItems];
         int neq = 0;
+        const int i0 = base + tid * kTopkItems;
+        const uint4 kv4 = i0 < NT ? keys4(i0) : make_uint4(0, 0, 0, 0);
+        const uint32_t kk[4] = {kv4.x, kv4.y, kv4.z, kv4.w};
 #pragma unroll
         for (int j = 0; j < kTopkItems; ++j) {
-            const int i = base + tid * kTopkItems + j;
+            const int i = i0 + j;
             gt[j] = eq[j] = false;
             if (i < NT) {
-                const uint32_t k = key_at(i);
-                gt[j] = k > thr;
-                eq[j] = k == thr;
+                gt[j] = kk[j] > thr;
+                eq[j] = kk[j] == thr;
             }
             neq += eq[j];
         }

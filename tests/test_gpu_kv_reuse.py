@@ -119,3 +119,31 @@ def test_stack4_reuse_equals_plain(ec):
 def test_stack40_reuse_equals_plain(ec):
     """The 40-layer Wan2.2-S2V-shaped stack, a full step and three cached steps."""
     _compare_stacks(ec, WAN_STACK40_32760, 4)
+
+
+def test_reuse_with_adaptive_rate_and_random_selection(ec):
+    """Reuse under a budget that changes from step to step (the adaptive rate
+    of Sec. 3.3) and under the Random selection ablation: still bit for bit."""
+    from paper_2608_02474_gb300.pipeline import AdaptiveRate, CachedStack
+    w = STACK4_7800
+    audio = torch.from_numpy(G.audio(w)).to(DEV)
+    cond = G.cond_tokens(w, G.audio(w))
+    blocks = [ec.DeviceBlock.from_host(G.block_weights(w, l), cond) for l in range(w.layers)]
+    xs = [bf(x) for x in G.step_inputs(w, G.latents(w), 6)]
+    for selection in ("energy", "random"):
+        outs, budgets = [], []
+        for reuse in (False, True):
+            st = CachedStack(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc, blocks, device=DEV,
+                             selection=selection, reuse_kv=reuse, seed=3)
+            st.set_audio(audio)
+            rate = AdaptiveRate(w.NT, 0.1, 0.5, 0.2, device=DEV)
+            ys = []
+            for t, x in enumerate(xs):
+                ys.append(st.step_adaptive(x, rate, full=t == 0).clone())
+            torch.cuda.synchronize()
+            assert ec.echo_get_device_error() == 0
+            outs.append(ys)
+            budgets.append(list(rate.budgets))
+        assert budgets[0] == budgets[1] and len(set(budgets[0])) > 1
+        for a, b in zip(*outs):
+            assert torch.equal(a, b), selection
