@@ -210,6 +210,13 @@ ECHO_DEV uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
     return r;
 }
 
+// 32-bit load from a shared::cluster address (this CTA's or another's).
+ECHO_DEV int ld_shared_cluster_s32(uint32_t cluster_addr) {
+    int v;
+    asm volatile("ld.shared::cluster.s32 %0, [%1];" : "=r"(v) : "r"(cluster_addr) : "memory");
+    return v;
+}
+
 // Arrive on an mbarrier given by its shared::cluster address (possibly another CTA's).
 ECHO_DEV void mbar_arrive_remote(uint32_t cluster_addr) {
     asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
@@ -248,7 +255,7 @@ ECHO_DEV bool mbar_wait_cluster(uint64_t *bar, uint32_t parity, volatile int *ab
     }
 }
 
-// All threads of both CTAs of the cluster.
+// All threads of every CTA of the cluster.
 ECHO_DEV void cluster_sync_all() {
     asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
                  "barrier.cluster.wait.acquire.aligned;" ::: "memory");

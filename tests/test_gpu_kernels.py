@@ -4,6 +4,8 @@ Bars: bit-exact for the int8 cache, scales, dequantised rows, drift scores and
 selected indices; rel <= 1e-5 for fp32 energies; bf16 outputs within the
 block tolerance (per-row normwise max rel <= 2e-2, mean rel <= 5e-3).
 """
+import os
+
 import numpy as np
 import pytest
 import torch
@@ -208,6 +210,60 @@ def test_select_with_and_without_workspace_agree(ec):
     for r in (a, b, c):
         assert np.array_equal(r.cpu().numpy(), oidx)
     no_device_error(ec)
+
+
+# Top-K alone (echo_select_random ranks caller keys): sizes around the split of
+# the keys over the CTAs of the cluster kernel (10240 keys and up, slices of at
+# most 51200 keys), the one-CTA kernel on either side, budgets of one key, of
+# all but one, and inside a run of equal keys that crosses slices.
+TOPK_SIZES = [(1, 4097), (1, 10239), (1, 10240), (1, 10241), (7, 4681), (21, 1560), (41, 1560),
+              (1, 65536), (3, 100001), (1, 409600), (1, 409601)]
+
+
+@pytest.mark.parametrize("T,N", TOPK_SIZES)
+@pytest.mark.parametrize("keys_kind", ["uniform", "three_levels", "one_level", "signed"])
+def test_topk_over_slices(ec, T, N, keys_kind):
+    NT = T * N
+    r = G.rng(NT + len(keys_kind))
+    if keys_kind == "uniform":
+        keys = r.random(NT, dtype=np.float32)
+    elif keys_kind == "three_levels":   # ties at every budget below, across slices
+        keys = np.floor(r.random(NT, dtype=np.float32) * 3).astype(F32)
+    elif keys_kind == "one_level":
+        keys = np.full(NT, 0.25, F32)
+    else:                               # negative and positive keys
+        keys = (r.random(NT, dtype=np.float32) - F32(0.5)) * F32(8)
+        keys[keys == 0] = F32(1)
+    kd = torch.from_numpy(keys).to(DEV)
+    for num, den in ((1, NT), (1, 20), (1, 2), (NT - 1, NT)):
+        idx, K = ec.echo_select_random(kd, T, N, num, den)
+        torch.cuda.synchronize()
+        assert K == oracle.select.refresh_budget(NT, num, den)
+        assert np.array_equal(idx.cpu().numpy(), oracle.select.random_subset(keys, K)), (num, den)
+    no_device_error(ec)
+
+
+@pytest.mark.parametrize("NT", [65536, 10920, 409600])
+def test_topk_first_call_in_a_process(ec, NT):
+    """The first top-K of a process, at a size whose keys need more dynamic
+    shared memory than the default cap leaves beside the kernel's own buffers."""
+    import subprocess
+    import sys
+    code = (
+        "import numpy as np, torch\n"
+        "from paper_2608_02474_gb300 import echocache as ec\n"
+        "import oracle\n"
+        f"NT = {NT}\n"
+        "keys = np.random.default_rng(NT).random(NT, dtype=np.float32)\n"
+        "idx, K = ec.echo_select_random(torch.from_numpy(keys).cuda(), 1, NT, 1, 5)\n"
+        "torch.cuda.synchronize()\n"
+        "assert ec.echo_get_device_error() == 0\n"
+        "assert np.array_equal(idx.cpu().numpy(), oracle.select.random_subset(keys, K))\n"
+        "print('ok')\n")
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([sys.executable, "-c", code], cwd=root, capture_output=True, text=True,
+                       timeout=300)
+    assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stdout + r.stderr
 
 
 def test_select_with_silence_is_drift_only(ec):

@@ -10,8 +10,9 @@ The test calls it through the C ABI twice in a row, on different inputs and
 sizes (the second call reuses the array the first one filled), and checks
 that each call selects exactly the indices echo_select selects with a
 workspace (indices are compared bit-exact, as in every selection test).
-A third case at 63960 tokens reaches the top-K path that keeps its keys in
-global memory and is also compared with the oracle's selection directly.
+A third case at 63960 tokens, near the static array's limit (its keys split
+over the 8-CTA cluster form of the top-K), is also compared with the oracle's
+selection directly.
 This file is collected last so that a failure here never hides another test.
 """
 import ctypes
@@ -70,11 +71,12 @@ def test_static_select_matches_workspace_select_on_two_calls(ec):
     assert ec.echo_get_device_error() == 0
 
 
-def test_static_select_keys_in_global_memory_match_the_oracle(ec):
-    """41 x 1560 = 63960 tokens (the 161-frame sweep shape, at a small width):
-    more keys than the top-K keeps in shared memory, so the selection keeps them
-    in global memory.  Two calls in a row (r = 1/20, then r = 1/2), each
-    compared bit for bit with echo_select and with the oracle's selection."""
+def test_static_select_near_the_size_limit_matches_the_oracle(ec):
+    """41 x 1560 = 63960 tokens (the 161-frame sweep shape, at a small width),
+    near the static array's 65536: more keys than one CTA holds in shared
+    memory, split over the CTAs of the cluster top-K.  Two calls in a row
+    (r = 1/20, then r = 1/2), each compared bit for bit with echo_select and
+    with the oracle's selection."""
     import oracle
     T, N, D = 41, 1560, 64
     x, q, s, e = _inputs(T, N, D, 21)
