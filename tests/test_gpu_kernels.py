@@ -375,13 +375,15 @@ ATTN_CASES = [
     (128, 64, 4, 128),
     (130, 672, 3, 128),
     (64, 7800, 2, 64),
-    # key sets up to 4096 take the persistent kernel (items chained per SM)
+    # key sets up to 2048 take the persistent kernel (items chained per SM)
     (6552, 672, 40, 128),    # cross-attention of the 32760-token block: 1040 items, 96-key blocks
     (3000, 160, 16, 64),     # 192 items (some CTAs take two), 96-key blocks with a masked tail
     (1000, 64, 4, 128),      # 64-key blocks
     (300, 32, 3, 64),        # 32-key blocks
-    (300, 4096, 2, 64),      # the largest key set of the persistent kernel
-    (300, 4097, 2, 64),      # one key more: the one-shot kernel
+    (300, 2048, 2, 128),     # the largest key set of the persistent kernel
+    (300, 2049, 2, 128),     # one key more: the one-shot kernel
+    (300, 4096, 2, 64),
+    (300, 4097, 2, 64),
 ]
 
 
