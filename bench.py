@@ -212,6 +212,8 @@ def roofline(records, K, peaks, timed_s=None):
                "peak": peak, "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
                "traffic": traffic, "algorithmic_flops": flops, "launch_ms": round(avg_ms, 4),
                "peak_source": source}
+        if "bf16_tflops_sustained" in peaks:   # beside it, always: the power-capped figure
+            out["frac_of_sustained"] = round(achieved / peaks["bf16_tflops_sustained"], 4)
     else:
         achieved = byts / (avg_ms * 1e-3) / 1e9
         peak = peaks["hbm_gbs"]

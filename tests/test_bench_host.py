@@ -123,6 +123,10 @@ def test_tensor_peak_follows_the_length_of_the_timed_region():
     assert bench.tensor_peak(PEAKS, bench.SUSTAINED_MIN_S)[0] == PEAKS["bf16_tflops_sustained"]
     out, _ = bench.roofline([("attention", 6552, 32760, 5120, 2.5)], 6552, PEAKS, timed_s=3.0)
     assert out["peak"] == PEAKS["bf16_tflops_sustained"] and "sustained" in out["peak_source"]
+    # the fraction of the power-capped peak is reported beside the rule's one
+    short, _ = bench.roofline([("attention", 6552, 32760, 5120, 2.5)], 6552, PEAKS, timed_s=0.13)
+    assert short["peak"] == PEAKS["bf16_tflops"]
+    assert short["frac_of_sustained"] == round(short["achieved"] / PEAKS["bf16_tflops_sustained"], 4)
 
 
 def test_both_arms_print_the_same_config():
