@@ -63,14 +63,14 @@ def gpu_layer(ec, blk, w, x, q, s, e, ratio, full=False):
     return idx.cpu().numpy(), y, qd, sd
 
 
-def check_active(g, o, emu, tag):
+def check_active(g, o, emu, tag, mean_bar=5e-3):
     """Normwise and mean bars, and the element-wise figure against the model's."""
     mx, mean = normwise_rel(g, o)
     el = elementwise_rel(g, o)
     el_m = elementwise_rel(emu, o)
     print(f"[{tag}] rows {len(o)}: normwise {mx:.3e}  mean {mean:.3e}  elementwise {el:.3e}  "
           f"(ideal bf16 {el_m:.3e}, ratio {el / el_m:.2f})")
-    assert mx <= 2e-2 and mean <= 5e-3, (tag, mx, mean)
+    assert mx <= 2e-2 and mean <= mean_bar, (tag, mx, mean, mean_bar)
     assert el <= EL_FACTOR * el_m, (tag, el, el_m)
     return mx, mean, el, el_m
 
@@ -123,7 +123,7 @@ def _trajectory(w, steps, layers, profile="speech"):
     return Ws, cond, e32, rec
 
 
-def _run_trajectory(ec, w, steps, layers, profile="speech", el_rows=256):
+def _run_trajectory(ec, w, steps, layers, profile="speech", el_rows=256, mean_vs_model=False):
     """Every (step, layer) of the oracle's trajectory; all active rows at the
     normwise and mean bars, and up to `el_rows` of them (half at random, half
     of highest score) for the element-wise comparison with the model."""
@@ -133,24 +133,32 @@ def _run_trajectory(ec, w, steps, layers, profile="speech", el_rows=256):
         g_idx, y, qd, sd = gpu_layer(ec, blks[l], w, x, q, s, e32, (w.ratio_num, w.ratio_den),
                                      full=t == 0)
         check_step(ec, w, Ws[l], cond, x, q, s, r, g_idx, y, qd, sd, f"{w.name} t={t} l={l}",
-                   el_rows)
+                   el_rows, mean_vs_model)
 
 
-def check_step(ec, w, W, cond, x, q, s, r, g_idx, y, qd, sd, tag, el_rows=256):
+def check_step(ec, w, W, cond, x, q, s, r, g_idx, y, qd, sd, tag, el_rows=256,
+               mean_vs_model=False):
     """One layer step against the oracle's result r on the same inputs: the
     indices, every active row at the normwise and mean bars, up to `el_rows`
     active rows (half at random, half of highest score) against the ideal bf16
-    model element-wise, the inactive rows and the cache write."""
+    model element-wise, the inactive rows and the cache write.  mean_vs_model
+    (rows wider than any of the paper's workloads, where the ideal bf16 block
+    itself is above 5e-3): the mean bar is 1.25 times the model's mean on the
+    same rows, every active row being compared with the model."""
     assert np.array_equal(g_idx, r.idx)
     g = y.float().cpu().numpy()
     mx, mean = normwise_rel(g[r.idx], r.y_act)
-    assert mx <= 2e-2 and mean <= 5e-3, (tag, mx, mean)
     j = np.arange(len(r.idx))
     if len(j) > el_rows:
+        assert not mean_vs_model, "the model's mean needs every active row"
         j = _sample_rows(j, r.scores[r.idx], n=el_rows // 2)
+    emu = M.block_active(x, r.idx[j], W, cond, w.H) if len(j) else None
+    mean_bar = 5e-3
+    if mean_vs_model and len(j):
+        mean_bar = max(mean_bar, 1.25 * normwise_rel(emu, r.y_act[j])[1])
+    assert mx <= 2e-2 and mean <= mean_bar, (tag, mx, mean, mean_bar)
     if len(j):
-        emu = M.block_active(x, r.idx[j], W, cond, w.H)
-        check_active(g[r.idx[j]], r.y_act[j], emu, tag)
+        check_active(g[r.idx[j]], r.y_act[j], emu, tag, mean_bar)
     check_cache_and_inactive(ec, w, r.idx, q, s, g, y, qd.cpu().numpy(), sd.cpu().numpy())
 
 
@@ -169,6 +177,21 @@ def test_stack4_every_step(ec):
 @pytest.mark.parametrize("profile", ["silence", "tone", "beats"])
 def test_tiny_profiles(ec, profile):
     _run_trajectory(ec, TINY_256, 3, 1, profile)
+
+
+@pytest.mark.parametrize("H,d", [(64, 128), (128, 64)])
+def test_widest_block_ragged_shapes(ec, H, d):
+    """The widest rows the ABI takes (D 8192), every other size ragged: 70
+    spatial latents per frame (210 tokens, divided by neither the 128-row
+    attention tile nor the 256-row GEMM tile), an FFN of 1088 (4.25 GEMM
+    N-tiles), 37 audio tokens (one masked key block), r = 1/3 (70 active
+    rows); the full step and one cached step."""
+    from dataclasses import replace
+    w = replace(TINY_256, name=f"widest_{H}x{d}", T=3, Hp=7, Wp=10, D=8192, H=H, d=d, F=1088,
+                Lc=37, n_samples=4800, ratio_num=1, ratio_den=3, steps=2, layers=1)
+    # at this width the ideal bf16 block's own mean relative error is about
+    # 8e-3 on these inputs (normwise max 1.1e-2): the mean is held against it
+    _run_trajectory(ec, w, 2, 1, mean_vs_model=True)
 
 
 def test_edge_ratios_and_aliasing(ec):
