@@ -219,6 +219,32 @@ def test_edge_ratios_and_aliasing(ec):
     assert ec.echo_get_device_error() == 0
 
 
+@pytest.mark.parametrize("which", ["first", "last", "middle", "all_but_one"])
+def test_one_active_row_and_all_but_one(ec, which):
+    """K = 1 (one query row through every GEMM and both attentions) and
+    K = NT - 1: an active row's output is the uncached block's at that row
+    (K and V always cover every token), every other row is the reconstructed
+    cache, and the cache holds the quantised rows returned."""
+    w = TINY_256
+    W = G.block_weights(w, 0)
+    cond = G.cond_tokens(w, G.audio(w))
+    x = G.latents(w)
+    q, s = oracle.cache.quantize_rows(G.step_input(w, x, 2))[:2]
+    blk = ec.DeviceBlock.from_host(W, cond)
+    dims = ec.BlockDims(w.T, w.N, w.D, w.H, w.d, w.F, w.Lc)
+    rows = {"first": [0], "last": [w.NT - 1], "middle": [w.NT // 2 + 3],
+            "all_but_one": [i for i in range(w.NT) if i != 77]}[which]
+    idx = np.asarray(rows, dtype=np.int32)
+    qd, sd = torch.from_numpy(q.copy()).to(DEV), torch.from_numpy(s.copy()).to(DEV)
+    y = ec.echo_block_step(blk, dims, bf(x), torch.from_numpy(idx).to(DEV), len(idx), qd, sd)
+    torch.cuda.synchronize()
+    assert ec.echo_get_device_error() == 0
+    g = y.float().cpu().numpy()
+    check_active(g[idx], oracle.block.uncached_block(x, W, cond, w.H)[idx],
+                 M.block_active(x, idx, W, cond, w.H), f"tiny K={len(idx)} {which}")
+    check_cache_and_inactive(ec, w, idx, q, s, g, y, qd.cpu().numpy(), sd.cpu().numpy())
+
+
 # ---------------------------------------------------------------------------
 # Full-size Wan2.2-S2V-shaped blocks (D 5120, 40 heads x 128, FFN 13824, 672
 # audio tokens).  The oracle recomputes K/V over every token and the block for

@@ -152,6 +152,8 @@ SELECT_CASES = [
     (2, 1000, 264, (1, 3), 0, False),
     (21, 1560, 5120, (1, 5), 0, True),
     (41, 1560, 128, (1, 20), 0, True),
+    (1, 300, 64, (1, 4), 0, True),      # one audio segment: its weight is 1
+    (1, 300, 64, (1, 4), 1, True),
 ]
 
 
