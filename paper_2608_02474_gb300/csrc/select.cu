@@ -196,6 +196,106 @@ ECHO_DEV int block_exclusive_scan(int v, int *warp_sums, int *total) {
     return r;
 }
 
+// Radix digits (bits [sh, sh + log2 nb)) of the n keys whose higher bits
+// equal `prefix` under `pmask`, counted into hist (zeroed by the caller).
+// keys4(i) returns keys i .. i + 3 (i a multiple of 4; keys at or past n are
+// ignored whatever they hold).
+template <typename KeyFn>
+ECHO_DEV void count_digits(KeyFn keys4, int n, int sh, int nb, uint32_t prefix, uint32_t pmask,
+                           int *hist) {
+    const int stride4 = blockDim.x * 4;
+    for (int b = threadIdx.x * 4; b < n; b += stride4 * 4) {
+        uint4 v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int i = b + u * stride4;
+            v[u] = i < n ? keys4(i) : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int i = b + u * stride4;
+            const uint32_t k[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                if (i + c < n && (k[c] & pmask) == prefix)
+                    atomicAdd(&hist[(k[c] >> sh) & (nb - 1)], 1);
+        }
+    }
+}
+
+// The digit that holds the krem-th largest counted key, the bins taken from
+// the highest down (thread t covers hi = nb-1-2t and hi-1); krem becomes that
+// key's rank within its bin.  Every thread returns the same digit.
+ECHO_DEV int pick_digit(const int *hist, int nb, int &krem, int *warp_sums, int *s_digit,
+                        int *s_krem) {
+    const int hi = nb - 1 - 2 * (int)threadIdx.x;
+    const int c_hi = hi >= 0 ? hist[hi] : 0;
+    const int c_lo = hi - 1 >= 0 ? hist[hi - 1] : 0;
+    int total;
+    const int above = block_exclusive_scan(c_hi + c_lo, warp_sums, &total);
+    if (hi >= 0 && above < krem && above + c_hi >= krem) {
+        *s_digit = hi;
+        *s_krem = krem - above;
+    }
+    if (hi - 1 >= 0 && above + c_hi < krem && above + c_hi + c_lo >= krem) {
+        *s_digit = hi - 1;
+        *s_krem = krem - above - c_hi;
+    }
+    __syncthreads();
+    const int digit = *s_digit;
+    krem = *s_krem;
+    __syncthreads();
+    return digit;
+}
+
+// Writes, in index order, the indices (first + i) of the n keys above thr and
+// of the keys equal to thr while fewer than need_eq of those have been taken.
+// eq_run and sel_run: keys equal to thr and keys taken before key 0 (by
+// lower-ranked slices); the first index written goes to idx[sel_run].
+template <typename KeyFn>
+ECHO_DEV void compact_in_index_order(KeyFn keys4, int n, int first, uint32_t thr, int need_eq,
+                                     int eq_run, int sel_run, int32_t *__restrict__ idx,
+                                     int *warp_sums) {
+    const int tile = kTopkThreads * kTopkItems;
+    for (int base = 0; base < n; base += tile) {
+        bool gt[kTopkItems], eq[kTopkItems];
+        int neq = 0;
+        const int i0 = base + (int)threadIdx.x * kTopkItems;
+        const uint4 kv4 = i0 < n ? keys4(i0) : make_uint4(0, 0, 0, 0);
+        const uint32_t kk[4] = {kv4.x, kv4.y, kv4.z, kv4.w};
+#pragma unroll
+        for (int j = 0; j < kTopkItems; ++j) {
+            const int i = i0 + j;
+            gt[j] = eq[j] = false;
+            if (i < n) {
+                gt[j] = kk[j] > thr;
+                eq[j] = kk[j] == thr;
+            }
+            neq += eq[j];
+        }
+        int eq_total;
+        int eq_before = eq_run + block_exclusive_scan(neq, warp_sums, &eq_total);
+        bool sel[kTopkItems];
+        int nsel = 0;
+#pragma unroll
+        for (int j = 0; j < kTopkItems; ++j) {
+            sel[j] = gt[j];
+            if (eq[j]) {
+                sel[j] = eq_before < need_eq;
+                ++eq_before;
+            }
+            nsel += sel[j];
+        }
+        int sel_total;
+        int pos = sel_run + block_exclusive_scan(nsel, warp_sums, &sel_total);
+#pragma unroll
+        for (int j = 0; j < kTopkItems; ++j)
+            if (sel[j]) idx[pos++] = first + i0 + j;
+        eq_run += eq_total;
+        sel_run += sel_total;
+    }
+}
+
 __global__ void __launch_bounds__(kTopkThreads)
 topk_kernel(const float *__restrict__ scores, int NT, int K, int keys_in_smem,
             int32_t *__restrict__ idx) {
@@ -254,88 +354,14 @@ topk_kernel(const float *__restrict__ scores, int NT, int K, int keys_in_smem,
         const int nb = 1 << widths[pass];
         for (int b = tid; b < 2048; b += blockDim.x) hist[b] = 0;
         __syncthreads();
-        for (int b = tid * 4; b < NT; b += stride4 * 4) {
-            uint4 v[4];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int i = b + u * stride4;
-                v[u] = i < NT ? keys4(i) : make_uint4(0, 0, 0, 0);
-            }
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int i = b + u * stride4;
-                const uint32_t k[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
-#pragma unroll
-                for (int c = 0; c < 4; ++c)
-                    if (i + c < NT && (k[c] & pmask) == prefix)
-                        atomicAdd(&hist[(k[c] >> sh) & (nb - 1)], 1);
-            }
-        }
+        count_digits(keys4, NT, sh, nb, prefix, pmask, hist);
         __syncthreads();
-        // thread t covers the two bins hi = nb-1-2t and lo = hi-1 (descending)
-        const int hi = nb - 1 - 2 * tid;
-        int c_hi = 0, c_lo = 0;
-        if (hi >= 0) c_hi = hist[hi];
-        if (hi - 1 >= 0) c_lo = hist[hi - 1];
-        int total;
-        const int above = block_exclusive_scan(c_hi + c_lo, warp_sums, &total);
-        if (hi >= 0 && above < krem && above + c_hi >= krem) {
-            s_digit = hi;
-            s_krem = krem - above;
-        }
-        if (hi - 1 >= 0 && above + c_hi < krem && above + c_hi + c_lo >= krem) {
-            s_digit = hi - 1;
-            s_krem = krem - above - c_hi;
-        }
-        __syncthreads();
-        prefix |= (uint32_t)s_digit << sh;
+        prefix |= (uint32_t)pick_digit(hist, nb, krem, warp_sums, &s_digit, &s_krem) << sh;
         pmask |= (uint32_t)(nb - 1) << sh;
-        krem = s_krem;
-        __syncthreads();
     }
     // prefix is the K-th largest key; take every larger key and the first
     // `krem` keys equal to it in index order.
-    const uint32_t thr = prefix;
-    const int need_eq = krem;
-    int eq_run = 0, sel_run = 0;
-    const int tile = kTopkThreads * kTopkItems;
-    for (int base = 0; base < NT; base += tile) {
-        bool gt[kTopkItems], eq[kTopkItems];
-        int neq = 0;
-        const int i0 = base + tid * kTopkItems;
-        const uint4 kv4 = i0 < NT ? keys4(i0) : make_uint4(0, 0, 0, 0);
-        const uint32_t kk[4] = {kv4.x, kv4.y, kv4.z, kv4.w};
-#pragma unroll
-        for (int j = 0; j < kTopkItems; ++j) {
-            const int i = i0 + j;
-            gt[j] = eq[j] = false;
-            if (i < NT) {
-                gt[j] = kk[j] > thr;
-                eq[j] = kk[j] == thr;
-            }
-            neq += eq[j];
-        }
-        int eq_total;
-        int eq_before = eq_run + block_exclusive_scan(neq, warp_sums, &eq_total);
-        bool sel[kTopkItems];
-        int nsel = 0;
-#pragma unroll
-        for (int j = 0; j < kTopkItems; ++j) {
-            sel[j] = gt[j];
-            if (eq[j]) {
-                sel[j] = eq_before < need_eq;
-                ++eq_before;
-            }
-            nsel += sel[j];
-        }
-        int sel_total;
-        int pos = sel_run + block_exclusive_scan(nsel, warp_sums, &sel_total);
-#pragma unroll
-        for (int j = 0; j < kTopkItems; ++j)
-            if (sel[j]) idx[pos++] = base + tid * kTopkItems + j;
-        eq_run += eq_total;
-        sel_run += sel_total;
-    }
+    compact_in_index_order(keys4, NT, 0, prefix, krem, 0, 0, idx, warp_sums);
 }
 
 constexpr int kTopkClusterCtas = 8;
@@ -415,6 +441,7 @@ topk_cluster_kernel(const float *__restrict__ scores, int NT, int K, int slice,
     }
     cluster_sync_all();   // every owner's buffers are zero before any CTA adds to them
 
+    auto keys4 = [&](int i) -> uint4 { return skeys4[i >> 2]; };
     uint32_t prefix = 0, pmask = 0;
     int krem = K;
     const int shifts[3] = {21, 10, 0};
@@ -424,23 +451,7 @@ topk_cluster_kernel(const float *__restrict__ scores, int NT, int K, int slice,
         const int nb = 1 << widths[pass];
         for (int b = tid; b < 2048; b += blockDim.x) hist[b] = 0;
         __syncthreads();
-        for (int b = tid * 4; b < n; b += stride4 * 4) {
-            uint4 v[4];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int i = b + u * stride4;
-                v[u] = i < n ? skeys4[i >> 2] : make_uint4(0, 0, 0, 0);
-            }
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int i = b + u * stride4;
-                const uint32_t k[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
-#pragma unroll
-                for (int c = 0; c < 4; ++c)
-                    if (i + c < n && (k[c] & pmask) == prefix)
-                        atomicAdd(&hist[(k[c] >> sh) & (nb - 1)], 1);
-            }
-        }
+        count_digits(keys4, n, sh, nb, prefix, pmask, hist);
         __syncthreads();
         for (int b = tid; b < nb; b += blockDim.x) {
             const int v = hist[b];
@@ -457,25 +468,8 @@ topk_cluster_kernel(const float *__restrict__ scores, int NT, int K, int slice,
             *reinterpret_cast<int4 *>(&full[b0]) = v;
         }
         __syncthreads();
-        // thread t covers the two bins hi = nb-1-2t and lo = hi-1 (descending)
-        const int hi = nb - 1 - 2 * tid;
-        const int c_hi = hi >= 0 ? full[hi] : 0;
-        const int c_lo = hi - 1 >= 0 ? full[hi - 1] : 0;
-        int total;
-        const int above = block_exclusive_scan(c_hi + c_lo, warp_sums, &total);
-        if (hi >= 0 && above < krem && above + c_hi >= krem) {
-            s_digit = hi;
-            s_krem = krem - above;
-        }
-        if (hi - 1 >= 0 && above + c_hi < krem && above + c_hi + c_lo >= krem) {
-            s_digit = hi - 1;
-            s_krem = krem - above - c_hi;
-        }
-        __syncthreads();
-        prefix |= (uint32_t)s_digit << sh;
+        prefix |= (uint32_t)pick_digit(full, nb, krem, warp_sums, &s_digit, &s_krem) << sh;
         pmask |= (uint32_t)(nb - 1) << sh;
-        krem = s_krem;
-        __syncthreads();
     }
     const uint32_t thr = prefix;
     const int need_eq = krem;
@@ -500,50 +494,13 @@ topk_cluster_kernel(const float *__restrict__ scores, int NT, int K, int slice,
         s_counts[1] = eq_total_slice;
     }
     cluster_sync_all();
-    int gt_before = 0, eq_run = 0;
+    int gt_before = 0, eq_before = 0;
     for (int r = 0; r < rank; ++r) {
         gt_before += ld_shared_cluster_s32(mapa_shared(smem_u32(&s_counts[0]), (uint32_t)r));
-        eq_run += ld_shared_cluster_s32(mapa_shared(smem_u32(&s_counts[1]), (uint32_t)r));
+        eq_before += ld_shared_cluster_s32(mapa_shared(smem_u32(&s_counts[1]), (uint32_t)r));
     }
-    int sel_run = gt_before + min(eq_run, need_eq);
-    const int tile = kTopkThreads * kTopkItems;
-    for (int base = 0; base < n; base += tile) {
-        bool gt[kTopkItems], eq[kTopkItems];
-        int neq = 0;
-        const int i0 = base + tid * kTopkItems;
-        const uint4 kv4 = i0 < n ? skeys4[i0 >> 2] : make_uint4(0, 0, 0, 0);
-        const uint32_t kk[4] = {kv4.x, kv4.y, kv4.z, kv4.w};
-#pragma unroll
-        for (int j = 0; j < kTopkItems; ++j) {
-            const int i = i0 + j;
-            gt[j] = eq[j] = false;
-            if (i < n) {
-                gt[j] = kk[j] > thr;
-                eq[j] = kk[j] == thr;
-            }
-            neq += eq[j];
-        }
-        int eq_total;
-        int eq_before = eq_run + block_exclusive_scan(neq, warp_sums, &eq_total);
-        bool sel[kTopkItems];
-        int nsel = 0;
-#pragma unroll
-        for (int j = 0; j < kTopkItems; ++j) {
-            sel[j] = gt[j];
-            if (eq[j]) {
-                sel[j] = eq_before < need_eq;
-                ++eq_before;
-            }
-            nsel += sel[j];
-        }
-        int sel_total;
-        int pos = sel_run + block_exclusive_scan(nsel, warp_sums, &sel_total);
-#pragma unroll
-        for (int j = 0; j < kTopkItems; ++j)
-            if (sel[j]) idx[pos++] = lo + i0 + j;
-        eq_run += eq_total;
-        sel_run += sel_total;
-    }
+    compact_in_index_order(keys4, n, lo, thr, need_eq, eq_before,
+                           gt_before + min(eq_before, need_eq), idx, warp_sums);
     cluster_sync_all();   // no CTA leaves while another may still read its counts
 }
 
