@@ -147,3 +147,30 @@ def test_reuse_with_adaptive_rate_and_random_selection(ec):
         assert budgets[0] == budgets[1] and len(set(budgets[0])) > 1
         for a, b in zip(*outs):
             assert torch.equal(a, b), selection
+
+
+def test_resume_with_reuse_matches_the_uninterrupted_run(ec, tmp_path):
+    """A stack with K/V kept across steps, its caches saved after three steps
+    and loaded into a fresh stack with reuse: the fresh stack recomputes every
+    K/V row on its first step and then follows the uninterrupted run bit for
+    bit, through steps where only the changed rows are recomputed."""
+    w = STACK4_7800
+    audio = torch.from_numpy(G.audio(w)).to(DEV)
+    cond = G.cond_tokens(w, G.audio(w))
+    blocks = [ec.DeviceBlock.from_host(G.block_weights(w, l), cond) for l in range(w.layers)]
+    xs = [bf(x) for x in G.step_inputs(w, G.latents(w), 7)]
+    a = _stack(ec, w, blocks, True)
+    a.set_audio(audio)
+    for t in range(3):
+        a.step(xs[t], w.ratio_num, w.ratio_den, full=t == 0)
+    path = str(tmp_path / "caches.pt")
+    a.save_caches(path)
+    b = _stack(ec, w, blocks, True)
+    b.set_audio(audio)
+    b.load_caches(path)
+    for t in range(3, 7):
+        ya = a.step(xs[t], w.ratio_num, w.ratio_den).clone()
+        yb = b.step(xs[t], w.ratio_num, w.ratio_den).clone()
+        torch.cuda.synchronize()
+        assert ec.echo_get_device_error() == 0
+        assert torch.equal(ya, yb), f"step {t}"
