@@ -154,7 +154,9 @@ echo_status run_active(const echo_block_weights *w, const echo_block_dims &d, co
     const __nv_bfloat16 *kvb = static_cast<const __nv_bfloat16 *>(kv);
     const __nv_bfloat16 *kvc = static_cast<const __nv_bfloat16 *>(w->KVc);
     echo_status s = ECHO_OK;
-    launch_rowmap(idx, K, NT, rowmap, st);
+    // the row map, and max |y_act| per row cleared for the FFN-down epilogue
+    uint32_t *amax = reinterpret_cast<uint32_t *>(ws + L.amax);
+    launch_rowmap(idx, K, NT, rowmap, amax, K, st);
     if (K > 0) {
         if (kv_ready) {
             launch_layernorm(x, ECHO_BF16, idx, K, D, na, st);   // the active rows only
@@ -186,9 +188,6 @@ echo_status run_active(const echo_block_weights *w, const echo_block_dims &d, co
                            ECHO_BF16}, st);
         if (s != ECHO_OK) return s;
         // the FFN-down epilogue also records max |y_act| per row for the cache write
-        uint32_t *amax = reinterpret_cast<uint32_t *>(ws + L.amax);
-        if (cudaMemsetAsync(amax, 0, sizeof(uint32_t) * (size_t)K, st) != cudaSuccess)
-            return ECHO_ERR_CUDA;
         LinearArgs down{u, d.F, K, d.F, w->W2, w->b2, D, 0, h2, ECHO_F32, nullptr,
                         y_scatter ? y_scatter : yact, D, ECHO_BF16};
         down.row_amax = amax;

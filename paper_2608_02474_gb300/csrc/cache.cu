@@ -128,9 +128,22 @@ dequant_kernel(const int8_t *__restrict__ q, const float *__restrict__ scale,
     }
 }
 
-__global__ void rowmap_kernel(const int32_t *__restrict__ idx, int K, int32_t *__restrict__ rowmap) {
-    const int j = blockIdx.x * blockDim.x + threadIdx.x;
-    if (j < K) rowmap[idx[j]] = j;
+// rowmap[i] = j where idx[j] == i, else -1: idx is ascending and distinct, so
+// each row binary-searches it (idx stays in L1/L2).  The first n_zero words of
+// `zero` are cleared in the same pass.
+__global__ void rowmap_kernel(const int32_t *__restrict__ idx, int K, int NT,
+                              int32_t *__restrict__ rowmap, uint32_t *__restrict__ zero,
+                              int n_zero) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n_zero) zero[i] = 0u;
+    if (i >= NT) return;
+    int lo = 0, hi = K;   // the first j with idx[j] >= i
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (__ldg(idx + mid) < i) lo = mid + 1;
+        else hi = mid;
+    }
+    rowmap[i] = (lo < K && __ldg(idx + lo) == i) ? lo : -1;
 }
 
 // y[i] = y_act[rowmap[i]] if rowmap[i] >= 0 else bf16(q[i] * s[i]); without
@@ -261,12 +274,12 @@ void launch_dequant(const int8_t *q, const float *scale, const int32_t *rows, in
                                                             static_cast<float *>(dst));
 }
 
-void launch_rowmap(const int32_t *idx, int32_t K, int32_t NT, int32_t *rowmap, cudaStream_t st) {
-    cudaMemsetAsync(rowmap, 0xFF, sizeof(int32_t) * (size_t)NT, st);
-    if (K > 0) {
-        LaunchScope ls(ECHO_K_ROWMAP, K, NT, 0, st);
-        rowmap_kernel<<<(K + 255) / 256, 256, 0, st>>>(idx, K, rowmap);
-    }
+void launch_rowmap(const int32_t *idx, int32_t K, int32_t NT, int32_t *rowmap, uint32_t *zero,
+                   int32_t n_zero, cudaStream_t st) {
+    const int n = NT > n_zero ? NT : n_zero;
+    if (n <= 0) return;
+    LaunchScope ls(ECHO_K_ROWMAP, K, NT, 0, st);
+    rowmap_kernel<<<(n + 255) / 256, 256, 0, st>>>(idx, K, NT, rowmap, zero, n_zero);
 }
 
 void launch_dequant_merge(const int8_t *q, const float *scale, const int32_t *rowmap,

@@ -68,7 +68,10 @@ void launch_quant(const void *src, echo_dtype st_t, const int32_t *rows, int32_t
                   int32_t D, int8_t *q, float *scale, cudaStream_t st);
 void launch_dequant(const int8_t *q, const float *scale, const int32_t *rows, int32_t n_rows,
                     int32_t D, void *dst, echo_dtype dt, cudaStream_t st);
-void launch_rowmap(const int32_t *idx, int32_t K, int32_t NT, int32_t *rowmap, cudaStream_t st);
+// rowmap[i] = position of token i in idx (ascending, distinct), else -1; also
+// clears zero[0 .. n_zero)
+void launch_rowmap(const int32_t *idx, int32_t K, int32_t NT, int32_t *rowmap, uint32_t *zero,
+                   int32_t n_zero, cudaStream_t st);
 void launch_dequant_merge(const int8_t *q, const float *scale, const int32_t *rowmap,
                           const void *y_act, int32_t NT, int32_t D, void *y, cudaStream_t st);
 // y[i] = bf16(q[i] s[i]) for rowmap[i] < 0; every other row of y (already the
